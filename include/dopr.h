@@ -1,0 +1,221 @@
+/*
+ * dopr.h -- C ABI of the GB300-native DoPR online scoring library (libdopr.so).
+ *
+ * DoPR (Sec. 3.1 "Problem Formulation", Sec. 3.3 "Offline Compression",
+ * Sec. 3.4 "Online Reranking") stores, for every document d, the multi-layer
+ * key/value states C~_d of K_infer = m compressed prefix positions.  Online,
+ * a pair (q, d) is scored by running the decoder over [q ; t_score] only,
+ * each layer attending to d's stored prefix keys/values before the causal
+ * online keys, and reading the score at t_score.  This library implements
+ * that online pass on one GPU: a device-resident prefix store, a batch
+ * packer that groups pairs by document, and the decoder kernels.
+ *
+ * Conventions for every entry point:
+ *   - Plain C types only.  bf16 tensors are passed as `const void*` to
+ *     16-bit bit patterns (IEEE bfloat16).  Matrices are row-major.
+ *   - Inputs are borrowed for the duration of the call; the library copies
+ *     what it keeps.  Outputs go to caller-owned buffers.  Library objects
+ *     are opaque and released by the matching *_destroy.
+ *   - Every argument is validated before any device work is launched; on an
+ *     error nothing is written to caller buffers and the object is left as
+ *     it was.  The status says what went wrong; dopr_last_error() returns a
+ *     thread-local message for the last failing call on this thread.
+ *   - Device work runs on the device that is current when the object is
+ *     created; use the same device for all calls on that object.
+ *   - Objects are not thread-safe: serialise calls on one object.
+ */
+#ifndef DOPR_H
+#define DOPR_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define DOPR_API __attribute__((visibility("default")))
+#else
+#define DOPR_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    DOPR_OK = 0,
+    DOPR_ERR_INVALID_ARG = 1,   /* bad pointer, size, index or shape          */
+    DOPR_ERR_UNKNOWN_DOC = 2,   /* a doc_id has no stored prefix              */
+    DOPR_ERR_INCOMPLETE = 3,    /* a weight or a doc layer was never supplied */
+    DOPR_ERR_OUT_OF_MEMORY = 4, /* device allocation or the store pool full   */
+    DOPR_ERR_CUDA = 5,          /* a CUDA runtime/driver call failed          */
+    DOPR_ERR_TIMEOUT = 6,       /* a bounded device wait ran out; the result
+                                   of that call is invalid, the context is not */
+    DOPR_ERR_UNSUPPORTED = 7    /* a shape this build does not handle         */
+} dopr_status;
+
+/*
+ * Decoder shape (Qwen3 family, the paper's backbone, Sec. 4.1).
+ * Supported: head_dim == 128; n_q_heads % n_kv_heads == 0;
+ * hidden % 256 == 0; ffn % 128 == 0; (n_q_heads + 2 n_kv_heads) * 128 % 256 == 0.
+ * score_token_id is t_score (Sec. 3.1), appended by the library to every
+ * query.  Positions m + j of online tokens must be < max_position.
+ */
+typedef struct {
+    int32_t n_layers;
+    int32_t hidden;
+    int32_t n_q_heads;
+    int32_t n_kv_heads;
+    int32_t head_dim;
+    int32_t ffn;
+    int32_t vocab;
+    int32_t score_token_id;
+    int32_t max_position;
+    float rope_theta;   /* RoPE base, rotate-half pairs (i, i + head_dim/2) */
+    float rms_eps;      /* RMSNorm epsilon                                  */
+} dopr_model_config;
+
+typedef struct dopr_model dopr_model;
+typedef struct dopr_store dopr_store;
+
+/* Weight kinds for dopr_model_put_weight; shapes are [rows][cols] bf16. */
+typedef enum {
+    DOPR_W_EMBED = 0,      /* [vocab][hidden]             (layer ignored) */
+    DOPR_W_ATTN_NORM = 1,  /* [hidden]      input RMSNorm gain            */
+    DOPR_W_Q = 2,          /* [n_q_heads*128][hidden]                     */
+    DOPR_W_K = 3,          /* [n_kv_heads*128][hidden]                    */
+    DOPR_W_V = 4,          /* [n_kv_heads*128][hidden]                    */
+    DOPR_W_Q_NORM = 5,     /* [128]         per-head RMSNorm gain on q    */
+    DOPR_W_K_NORM = 6,     /* [128]         per-head RMSNorm gain on k    */
+    DOPR_W_O = 7,          /* [hidden][n_q_heads*128]                     */
+    DOPR_W_MLP_NORM = 8,   /* [hidden]      post-attention RMSNorm gain   */
+    DOPR_W_GATE = 9,       /* [ffn][hidden]                               */
+    DOPR_W_UP = 10,        /* [ffn][hidden]                               */
+    DOPR_W_DOWN = 11,      /* [hidden][ffn]                               */
+    DOPR_W_FINAL_NORM = 12,/* [hidden]                    (layer ignored) */
+    DOPR_W_SCORE_HEAD = 13 /* [2][hidden]: row 0 "yes", row 1 "no"
+                              (layer ignored)                             */
+} dopr_weight_kind;
+
+/* Create a model: allocates device memory for all weights of `cfg` (left
+ * unset until put).  *out receives the handle.  Errors: INVALID_ARG,
+ * UNSUPPORTED, OUT_OF_MEMORY, CUDA. */
+DOPR_API dopr_status dopr_model_create(const dopr_model_config *cfg, dopr_model **out);
+
+/* Copy one weight tensor into the model (converted to the library's own
+ * device layout).  `src` holds n_elems bf16 values in the layout listed
+ * under dopr_weight_kind; src_on_device != 0 means `src` is a device
+ * pointer.  Re-putting a weight replaces it.  Synchronous.
+ * Errors: INVALID_ARG (kind, layer or n_elems wrong), CUDA. */
+DOPR_API dopr_status dopr_model_put_weight(dopr_model *model, int32_t kind, int32_t layer, const void *src,
+                                  int64_t n_elems, int32_t src_on_device);
+
+/* Release a model and its device memory.  NULL is accepted. */
+DOPR_API dopr_status dopr_model_destroy(dopr_model *model);
+
+/*
+ * Prefix store (Sec. 3.3: the offline store of C~_d; Sec. 3.4: fetched per
+ * candidate).  Holds doc ids 0..max_doc_id in a device pool of pool_bytes
+ * bytes; each document takes dopr_prefix_bytes(cfg, m) bytes of it.
+ * Errors: INVALID_ARG, UNSUPPORTED, OUT_OF_MEMORY, CUDA.
+ */
+DOPR_API dopr_status dopr_store_create(const dopr_model_config *cfg, int64_t max_doc_id, int64_t pool_bytes,
+                              dopr_store **out);
+
+/*
+ * Store one layer of a document's compressed prefix states (Sec. 3.4 and
+ * its footnote: the multi-layer K/V obtained by forwarding the selected
+ * representations as prefix inputs).
+ *   k, v: bf16 [m][n_kv_heads][head_dim].  k is the key after the per-head
+ *         RMSNorm and after RoPE at positions 0..m-1; v is the raw value.
+ *   0 <= m <= 256 (the largest K_infer of the paper's settings, Tab. 8);
+ *   m == 0 stores an empty prefix (the pass then equals a query-only forward).
+ * The first put of a doc reserves its block; later puts must give the same
+ * m (a different m is INVALID_ARG) and replace that layer.  A doc can be
+ * scored once all n_layers layers were put.  Synchronous.
+ * Errors: INVALID_ARG, OUT_OF_MEMORY (pool full), CUDA.
+ */
+DOPR_API dopr_status dopr_store_put(dopr_store *store, int64_t doc_id, int32_t m, int32_t layer, const void *k,
+                           const void *v, int32_t src_on_device);
+
+/* Release a store.  NULL is accepted. */
+DOPR_API dopr_status dopr_store_destroy(dopr_store *store);
+
+/* Bytes of stored prefix state for one document of m prefix positions:
+ * m * n_layers * 2 (K,V) * n_kv_heads * head_dim * 2 bytes.  This is the
+ * document-side memory figure of Tab. 3 / Tab. 9.  Returns -1 on a bad cfg. */
+DOPR_API int64_t dopr_prefix_bytes(const dopr_model_config *cfg, int32_t m);
+
+/*
+ * Score a batch of (query, document) pairs (Sec. 3.4).
+ *   q_offsets [n_pairs+1] int32: query p is q_tokens[q_offsets[p] .. q_offsets[p+1]);
+ *             q_offsets[0] == 0, non-decreasing; empty queries are allowed
+ *             (the pair is then scored on the score token alone).
+ *   q_tokens  int32 token ids in [0, vocab).
+ *   doc_ids   [n_pairs] int64, each with a complete prefix in `store`.
+ *   scores    [n_pairs] float, written in input order: the "yes" minus
+ *             "no" logit at the score token.
+ *   cuda_stream: a cudaStream_t, or NULL for the default stream.
+ *   io_on_device: 0 = the four arrays are host memory (copied in and out by
+ *             the call); 1 = device memory (read and written in place).
+ * The call is synchronous in both modes: it synchronises `cuda_stream`
+ * once after packing (to size the launches) and once at the end, then
+ * reports the device error word.  Pairs of one doc_id are grouped so that
+ * their prefix is staged once per group; scores do not depend on batch
+ * order.  With io_on_device = 1 the inputs are validated on the device and
+ * an invalid batch returns its error before any decoder kernel runs.
+ * Errors: INVALID_ARG, UNKNOWN_DOC, INCOMPLETE, OUT_OF_MEMORY, CUDA, TIMEOUT.
+ */
+DOPR_API dopr_status dopr_score(dopr_model *model, dopr_store *store, int32_t n_pairs, const int32_t *q_offsets,
+                       const int32_t *q_tokens, const int64_t *doc_ids, float *scores, void *cuda_stream,
+                       int32_t io_on_device);
+
+/*
+ * The packing plan dopr_score uses (its device packer), copied to host
+ * arrays, for testing.  Inputs as in dopr_score (host memory).  Outputs,
+ * all host int32:
+ *   perm     [n_pairs]    input index of the pair in sorted position s;
+ *                         pairs are ordered by (doc_id, input index)
+ *   tok_off  [n_pairs+1]  first packed token of sorted pair s
+ *   tok_pos  [T]          RoPE position of packed token t (m_doc + j)
+ *   tok_id   [T]          token id of packed token t (score token last)
+ *   tok_pair [T]          sorted pair index of packed token t
+ * with T = q_offsets[n_pairs] - q_offsets[0] + n_pairs.
+ * Errors: as dopr_score.
+ */
+DOPR_API dopr_status dopr_debug_pack_plan(dopr_model *model, dopr_store *store, int32_t n_pairs, const int32_t *q_offsets,
+                                 const int32_t *q_tokens, const int64_t *doc_ids, int32_t *perm, int32_t *tok_off,
+                                 int32_t *tok_pos, int32_t *tok_id, int32_t *tok_pair);
+
+/*
+ * The dense projection kernel alone, for testing: C = A * B^T with A bf16
+ * [M][K], B bf16 [N][K] (device pointers), fp32 accumulation.
+ *   epilogue 0: out bf16 [M][N] = C
+ *   epilogue 1: out fp32 [M][N] += C            (residual add)
+ *   epilogue 2: out bf16 [M][N/2] = silu(G) * U, where B's rows come in
+ *               blocks of 256: rows 256b..256b+127 are gate rows 128b.., rows
+ *               256b+128..256b+255 the matching up rows (SwiGLU, Sec. 4.1 backbone)
+ * Requires K % 64 == 0 and N % 256 == 0.  Runs on cuda_stream (NULL = default)
+ * and returns after completion.  Errors: INVALID_ARG, UNSUPPORTED, CUDA, TIMEOUT.
+ */
+DOPR_API dopr_status dopr_debug_gemm(int32_t M, int32_t N, int32_t K, const void *A, const void *B, void *out,
+                            int32_t epilogue, void *cuda_stream);
+
+/*
+ * Runs one test kernel whose bounded wait on a barrier that nothing
+ * completes must give up after about timeout_ms milliseconds.  Returns
+ * DOPR_ERR_TIMEOUT when the kernel reported the expired wait (the expected
+ * result), DOPR_OK if it did not.  Used to check the timeout path of the
+ * device waits without hanging the GPU.
+ */
+DOPR_API dopr_status dopr_debug_wait_timeout(int32_t timeout_ms);
+
+/* Thread-local message describing the last failed call on this thread
+ * ("" if none).  The pointer stays valid until the next call on the thread. */
+DOPR_API const char *dopr_last_error(void);
+
+/* Library version string. */
+DOPR_API const char *dopr_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DOPR_H */

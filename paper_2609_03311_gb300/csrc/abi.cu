@@ -1,0 +1,782 @@
+// abi.cu -- C ABI of libdopr (include/dopr.h): the model and prefix-store
+// objects, host-side validation, and the engine that runs the online scoring
+// pass (DoPR Sec. 3.4) as a sequence of sm_103a kernels on the caller's stream.
+//
+// Engine of dopr_score:
+//   1. validate (host inputs on the host; device inputs in the packer kernel);
+//   2. device packer part 1: stable sort by doc id, packed token offsets;
+//   3. one small device->host read (offsets, slots, error word) to size launches;
+//   4. host splits the sorted pairs into chunks of whole pairs (<= chunk_cap
+//      tokens) and each chunk into attention work items (runs of <= 8 pairs of
+//      one document); packer part 2 writes token ids and positions;
+//   5. per chunk: embed+norm, then per layer QKV GEMM, QK-norm+RoPE, attention
+//      over prefix + causal keys, O GEMM (+residual), norm, gate/up GEMM
+//      (+SwiGLU), down GEMM (+residual), next norm; finally the score head,
+//      which scatters scores to input order.
+#include <cudaTypedefs.h>
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "device_common.cuh"
+#include "internal.h"
+
+struct dopr_model : dopr::Model {};
+struct dopr_store : dopr::Store {};
+
+namespace dopr {
+namespace {
+
+thread_local std::string g_last_error;
+
+dopr_status fail(dopr_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+#define CUDA_TRY(call)                                                                            \
+  do {                                                                                            \
+    cudaError_t e_ = (call);                                                                      \
+    if (e_ != cudaSuccess)                                                                        \
+      return fail(e_ == cudaErrorMemoryAllocation ? DOPR_ERR_OUT_OF_MEMORY : DOPR_ERR_CUDA,       \
+                  "%s failed: %s (%s:%d)", #call, cudaGetErrorString(e_), __FILE__, __LINE__);   \
+  } while (0)
+
+#define STATUS_TRY(call)            \
+  do {                              \
+    dopr_status s_ = (call);        \
+    if (s_ != DOPR_OK) return s_;   \
+  } while (0)
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+dopr_status check_cfg(const dopr_model_config* c) {
+  if (!c) return fail(DOPR_ERR_INVALID_ARG, "config is NULL");
+  if (c->n_layers <= 0 || c->hidden <= 0 || c->n_q_heads <= 0 || c->n_kv_heads <= 0 || c->ffn <= 0 ||
+      c->vocab <= 0 || c->max_position <= 0)
+    return fail(DOPR_ERR_INVALID_ARG, "config sizes must be positive");
+  if (c->score_token_id < 0 || c->score_token_id >= c->vocab)
+    return fail(DOPR_ERR_INVALID_ARG, "score_token_id %d outside [0, vocab)", c->score_token_id);
+  if (!(c->rope_theta > 0.f) || !(c->rms_eps >= 0.f)) return fail(DOPR_ERR_INVALID_ARG, "bad rope_theta / rms_eps");
+  if (c->head_dim != HEAD_DIM) return fail(DOPR_ERR_UNSUPPORTED, "head_dim must be 128 (got %d)", c->head_dim);
+  if (c->n_q_heads % c->n_kv_heads) return fail(DOPR_ERR_UNSUPPORTED, "n_q_heads must be a multiple of n_kv_heads");
+  const int G = c->n_q_heads / c->n_kv_heads;
+  if (16 % G != 0 && G % 16 != 0) return fail(DOPR_ERR_UNSUPPORTED, "GQA group size %d not supported", G);
+  if (c->hidden % GEMM_BN) return fail(DOPR_ERR_UNSUPPORTED, "hidden must be a multiple of 256");
+  if (c->ffn % 128) return fail(DOPR_ERR_UNSUPPORTED, "ffn must be a multiple of 128");
+  if (((c->n_q_heads + 2 * c->n_kv_heads) * HEAD_DIM) % GEMM_BN)
+    return fail(DOPR_ERR_UNSUPPORTED, "(n_q_heads + 2 n_kv_heads) * 128 must be a multiple of 256");
+  if ((c->n_q_heads * HEAD_DIM) % GEMM_BK) return fail(DOPR_ERR_UNSUPPORTED, "n_q_heads * 128 % 64");
+  if (c->max_position > (1 << 20)) return fail(DOPR_ERR_UNSUPPORTED, "max_position above 2^20");
+  return DOPR_OK;
+}
+
+template <typename T>
+dopr_status dev_alloc(T** p, size_t count) {
+  *p = nullptr;
+  if (count == 0) return DOPR_OK;
+  CUDA_TRY(cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T)));
+  return DOPR_OK;
+}
+template <typename T>
+void dev_free(T*& p) {
+  if (p) cudaFree(p);
+  p = nullptr;
+}
+template <typename T>
+dopr_status host_alloc(T** p, size_t count) {
+  *p = nullptr;
+  if (count == 0) return DOPR_OK;
+  CUDA_TRY(cudaMallocHost(reinterpret_cast<void**>(p), count * sizeof(T)));
+  return DOPR_OK;
+}
+template <typename T>
+void host_free(T*& p) {
+  if (p) cudaFreeHost(p);
+  p = nullptr;
+}
+
+int32_t kind_count() { return DOPR_W_SCORE_HEAD + 1; }
+bool kind_is_global(int32_t k) {
+  return k == DOPR_W_EMBED || k == DOPR_W_FINAL_NORM || k == DOPR_W_SCORE_HEAD;
+}
+
+void free_workspace(Workspace& w) {
+  dev_free(w.r); dev_free(w.xn); dev_free(w.qkv); dev_free(w.o); dev_free(w.act);
+  dev_free(w.q_off); dev_free(w.q_tok); dev_free(w.doc_ids); dev_free(w.scores);
+  dev_free(w.pair_slot); dev_free(w.perm); dev_free(w.sorted_slot); dev_free(w.tok_off);
+  dev_free(w.tok_id); dev_free(w.tok_pos); dev_free(w.tok_pair); dev_free(w.doc_count);
+  dev_free(w.items); dev_free(w.err);
+  host_free(w.h_tok_off); host_free(w.h_sorted_slot); host_free(w.h_err); host_free(w.h_items);
+  w = Workspace{};
+}
+
+void free_model(Model* m) {
+  dev_free(m->embed); dev_free(m->attn_norm); dev_free(m->w_qkv); dev_free(m->q_norm); dev_free(m->k_norm);
+  dev_free(m->w_o); dev_free(m->mlp_norm); dev_free(m->w_gu); dev_free(m->w_down); dev_free(m->final_norm);
+  dev_free(m->score_head); dev_free(m->rope);
+  free_workspace(m->ws);
+}
+
+void free_store(Store* s) {
+  dev_free(s->pool); dev_free(s->d_slot_of); dev_free(s->d_slot_m); dev_free(s->d_slot_row); dev_free(s->d_slot_ok);
+}
+
+dopr_status build_weight_maps(Model* m) {
+  const auto& c = m->cfg;
+  const int H = c.hidden, F = c.ffn, L = c.n_layers;
+  m->tm_qkv.resize(L); m->tm_o.resize(L); m->tm_gu.resize(L); m->tm_down.resize(L);
+  for (int l = 0; l < L; ++l) {
+    bool ok = make_tmap_bf16_2d(&m->tm_qkv[l], m->w_qkv + (size_t)l * m->qkv_dim * H, H, m->qkv_dim, (uint64_t)H * 2,
+                                GEMM_BK, GEMM_BN, true) &&
+              make_tmap_bf16_2d(&m->tm_o[l], m->w_o + (size_t)l * H * m->o_dim, m->o_dim, H, (uint64_t)m->o_dim * 2,
+                                GEMM_BK, GEMM_BN, true) &&
+              make_tmap_bf16_2d(&m->tm_gu[l], m->w_gu + (size_t)l * 2 * F * H, H, 2 * F, (uint64_t)H * 2, GEMM_BK,
+                                GEMM_BN, true) &&
+              make_tmap_bf16_2d(&m->tm_down[l], m->w_down + (size_t)l * H * F, F, H, (uint64_t)F * 2, GEMM_BK,
+                                GEMM_BN, true);
+    if (!ok) return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for layer %d weights", l);
+  }
+  m->maps_ok = true;
+  return DOPR_OK;
+}
+
+dopr_status alloc_chunk_buffers(Model* m, int cap) {
+  const auto& c = m->cfg;
+  Workspace& w = m->ws;
+  w.chunk_cap = cap;
+  STATUS_TRY(dev_alloc(&w.r, (size_t)cap * c.hidden));
+  STATUS_TRY(dev_alloc(&w.xn, (size_t)cap * c.hidden));
+  STATUS_TRY(dev_alloc(&w.qkv, (size_t)cap * m->qkv_dim));
+  STATUS_TRY(dev_alloc(&w.o, (size_t)cap * m->o_dim));
+  STATUS_TRY(dev_alloc(&w.act, (size_t)cap * c.ffn));
+  STATUS_TRY(dev_alloc(&w.err, 1));
+  STATUS_TRY(host_alloc(&w.h_err, 1));
+  bool ok = make_tmap_bf16_2d(&w.tm_xn, w.xn, c.hidden, cap, (uint64_t)c.hidden * 2, GEMM_BK, GEMM_BM, true) &&
+            make_tmap_bf16_2d(&w.tm_o, w.o, m->o_dim, cap, (uint64_t)m->o_dim * 2, GEMM_BK, GEMM_BM, true) &&
+            make_tmap_bf16_2d(&w.tm_act, w.act, c.ffn, cap, (uint64_t)c.ffn * 2, GEMM_BK, GEMM_BM, true);
+  if (!ok) return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for activation buffers");
+  return DOPR_OK;
+}
+
+// Grow the per-call buffers.
+dopr_status ensure_call_buffers(Model* m, int64_t n_pairs, int64_t n_tokens, int64_t n_qtokens, int64_t n_docs) {
+  Workspace& w = m->ws;
+  if (n_pairs > w.pair_cap) {
+    const int64_t cap = std::max<int64_t>(n_pairs, 2 * w.pair_cap);
+    dev_free(w.q_off); dev_free(w.doc_ids); dev_free(w.scores); dev_free(w.pair_slot); dev_free(w.perm);
+    dev_free(w.sorted_slot); dev_free(w.tok_off); dev_free(w.items);
+    STATUS_TRY(dev_alloc(&w.q_off, cap + 1));
+    STATUS_TRY(dev_alloc(&w.doc_ids, cap));
+    STATUS_TRY(dev_alloc(&w.scores, cap));
+    STATUS_TRY(dev_alloc(&w.pair_slot, cap));
+    STATUS_TRY(dev_alloc(&w.perm, cap));
+    STATUS_TRY(dev_alloc(&w.sorted_slot, cap));
+    STATUS_TRY(dev_alloc(&w.tok_off, cap + 1));
+    STATUS_TRY(dev_alloc(&w.items, cap + 1024));
+    w.pair_cap = cap;
+    w.item_cap = cap + 1024;
+  }
+  if (n_pairs > w.h_pair_cap) {
+    const int64_t cap = std::max<int64_t>(n_pairs, 2 * w.h_pair_cap);
+    host_free(w.h_tok_off); host_free(w.h_sorted_slot); host_free(w.h_items);
+    STATUS_TRY(host_alloc(&w.h_tok_off, cap + 1));
+    STATUS_TRY(host_alloc(&w.h_sorted_slot, cap));
+    STATUS_TRY(host_alloc(&w.h_items, cap + 1024));
+    w.h_pair_cap = cap;
+    w.h_item_cap = cap + 1024;
+  }
+  if (n_tokens > w.tok_cap) {
+    const int64_t cap = std::max<int64_t>(n_tokens, 2 * w.tok_cap);
+    dev_free(w.tok_id); dev_free(w.tok_pos); dev_free(w.tok_pair);
+    STATUS_TRY(dev_alloc(&w.tok_id, cap));
+    STATUS_TRY(dev_alloc(&w.tok_pos, cap));
+    STATUS_TRY(dev_alloc(&w.tok_pair, cap));
+    w.tok_cap = cap;
+  }
+  if (n_qtokens > w.qtok_cap) {
+    const int64_t cap = std::max<int64_t>(n_qtokens, 2 * w.qtok_cap);
+    dev_free(w.q_tok);
+    STATUS_TRY(dev_alloc(&w.q_tok, cap));
+    w.qtok_cap = cap;
+  }
+  if (n_docs > w.doc_cap) {
+    dev_free(w.doc_count);
+    STATUS_TRY(dev_alloc(&w.doc_count, n_docs));
+    w.doc_cap = n_docs;
+  }
+  return DOPR_OK;
+}
+
+dopr_status map_device_error(int e) {
+  if (e & DEV_ERR_TIMEOUT) return fail(DOPR_ERR_TIMEOUT, "a bounded device wait timed out");
+  if (e & DEV_ERR_UNKNOWN_DOC) return fail(DOPR_ERR_UNKNOWN_DOC, "a doc_id has no stored prefix");
+  if (e & DEV_ERR_INCOMPLETE) return fail(DOPR_ERR_INCOMPLETE, "a doc is missing stored layers");
+  if (e & DEV_ERR_BAD_TOKEN) return fail(DOPR_ERR_INVALID_ARG, "a token id is outside [0, vocab)");
+  if (e & DEV_ERR_BAD_OFFSETS) return fail(DOPR_ERR_INVALID_ARG, "q_offsets must start at 0 and not decrease");
+  if (e & DEV_ERR_POSITION) return fail(DOPR_ERR_INVALID_ARG, "m + query length + 1 exceeds max_position");
+  return DOPR_OK;
+}
+
+bool same_shape(const dopr_model_config& a, const dopr_model_config& b) {
+  return a.n_layers == b.n_layers && a.n_kv_heads == b.n_kv_heads && a.head_dim == b.head_dim;
+}
+
+// Host validation of host-resident inputs (before any launch).
+dopr_status validate_host_inputs(const Model* m, const Store* s, int32_t n, const int32_t* qo, const int32_t* qt,
+                                 const int64_t* doc) {
+  if (qo[0] != 0) return fail(DOPR_ERR_INVALID_ARG, "q_offsets[0] must be 0");
+  for (int32_t p = 0; p < n; ++p) {
+    const int32_t L = qo[p + 1] - qo[p];
+    if (L < 0) return fail(DOPR_ERR_INVALID_ARG, "q_offsets decreases at pair %d", p);
+    const int64_t d = doc[p];
+    if (d < 0 || d > s->max_doc_id || s->slot_of[d] < 0)
+      return fail(DOPR_ERR_UNKNOWN_DOC, "pair %d: doc_id %lld has no stored prefix", p, (long long)d);
+    const int32_t slot = s->slot_of[d];
+    if (!s->slot_ok[slot]) return fail(DOPR_ERR_INCOMPLETE, "pair %d: doc_id %lld is missing layers", p, (long long)d);
+    if ((int64_t)s->slot_m[slot] + L + 1 > m->cfg.max_position)
+      return fail(DOPR_ERR_INVALID_ARG, "pair %d: m + query length + 1 exceeds max_position", p);
+  }
+  const int64_t nt = qo[n];
+  for (int64_t i = 0; i < nt; ++i)
+    if (qt[i] < 0 || qt[i] >= m->cfg.vocab)
+      return fail(DOPR_ERR_INVALID_ARG, "q_tokens[%lld] = %d outside [0, vocab)", (long long)i, qt[i]);
+  return DOPR_OK;
+}
+
+// The packer's device arguments for one call.
+PackArgs pack_args(Model* m, Store* s, int32_t n, const int32_t* dqo, const int32_t* dqt, const int64_t* ddoc) {
+  Workspace& w = m->ws;
+  PackArgs a{};
+  a.n_pairs = n;
+  a.q_off = dqo;
+  a.q_tok = dqt;
+  a.doc_ids = ddoc;
+  a.max_doc_id = s->max_doc_id;
+  a.slot_of = s->d_slot_of;
+  a.slot_m = s->d_slot_m;
+  a.slot_ok = s->d_slot_ok;
+  a.vocab = m->cfg.vocab;
+  a.score_token = m->cfg.score_token_id;
+  a.max_position = m->cfg.max_position;
+  a.doc_count = w.doc_count;
+  a.pair_slot = w.pair_slot;
+  a.perm = w.perm;
+  a.sorted_slot = w.sorted_slot;
+  a.tok_off = w.tok_off;
+  a.tok_id = w.tok_id;
+  a.tok_pos = w.tok_pos;
+  a.tok_pair = w.tok_pair;
+  a.err = w.err;
+  return a;
+}
+
+struct Plan {
+  int64_t n_tokens = 0;
+  std::vector<int32_t> chunk_pair;  // chunk c covers sorted pairs [chunk_pair[c], chunk_pair[c+1])
+  std::vector<int32_t> chunk_item;  // and attention items [chunk_item[c], chunk_item[c+1])
+  int32_t n_items = 0;
+};
+
+// Steps 1-4 of the engine.  Inputs are device pointers.  On return the packed
+// plan is on the device and the chunking in `plan`.
+dopr_status run_packer(Model* m, Store* s, int32_t n, const int32_t* dqo, const int32_t* dqt, const int64_t* ddoc,
+                       cudaStream_t st, Plan& plan) {
+  Workspace& w = m->ws;
+  CUDA_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), st));
+  PackArgs a = pack_args(m, s, n, dqo, dqt, ddoc);
+  CUDA_TRY(launch_pack_order(a, st));
+  CUDA_TRY(cudaMemcpyAsync(w.h_tok_off, w.tok_off, sizeof(int32_t) * (n + 1), cudaMemcpyDeviceToHost, st));
+  CUDA_TRY(cudaMemcpyAsync(w.h_sorted_slot, w.sorted_slot, sizeof(int32_t) * n, cudaMemcpyDeviceToHost, st));
+  CUDA_TRY(cudaMemcpyAsync(w.h_err, w.err, sizeof(int), cudaMemcpyDeviceToHost, st));
+  CUDA_TRY(cudaStreamSynchronize(st));
+  STATUS_TRY(map_device_error(*w.h_err));
+  plan.n_tokens = w.h_tok_off[n];
+  // token buffers sized from the packed total, then packer part 2
+  STATUS_TRY(ensure_call_buffers(m, n, plan.n_tokens, 0, 0));
+  a = pack_args(m, s, n, dqo, dqt, ddoc);
+  CUDA_TRY(launch_pack_tokens(a, st));
+  // chunks of whole pairs, then attention items (runs of one doc, <= ATTN_MAX_PAIRS)
+  const int cap = w.chunk_cap;
+  plan.chunk_pair.assign(1, 0);
+  plan.chunk_item.assign(1, 0);
+  int32_t items = 0;
+  int32_t s0 = 0;
+  while (s0 < n) {
+    int32_t s1 = s0 + 1;
+    if (w.h_tok_off[s1] - w.h_tok_off[s0] > cap)
+      return fail(DOPR_ERR_UNSUPPORTED, "one pair has more tokens than a chunk (%d)", cap);
+    while (s1 < n && w.h_tok_off[s1 + 1] - w.h_tok_off[s0] <= cap) ++s1;
+    int32_t i = s0;
+    while (i < s1) {
+      int32_t j = i + 1;
+      while (j < s1 && j - i < ATTN_MAX_PAIRS && w.h_sorted_slot[j] == w.h_sorted_slot[i]) ++j;
+      AttnItem it;
+      it.pair_begin = i;
+      it.pair_end = j;
+      it.slot = w.h_sorted_slot[i];
+      it.m = s->slot_m[it.slot];
+      w.h_items[items++] = it;
+      i = j;
+    }
+    plan.chunk_pair.push_back(s1);
+    plan.chunk_item.push_back(items);
+    s0 = s1;
+  }
+  plan.n_items = items;
+  if (items > 0) CUDA_TRY(cudaMemcpyAsync(w.items, w.h_items, sizeof(AttnItem) * items, cudaMemcpyHostToDevice, st));
+  return DOPR_OK;
+}
+
+dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cudaStream_t st) {
+  Workspace& w = m->ws;
+  const auto& c = m->cfg;
+  const int H = c.hidden, F = c.ffn, L = c.n_layers;
+  const int mpad = ((s->max_m + 63) / 64) * 64;
+  for (size_t ci = 0; ci + 1 < plan.chunk_pair.size(); ++ci) {
+    const int32_t s0 = plan.chunk_pair[ci], s1 = plan.chunk_pair[ci + 1];
+    const int32_t t0 = w.h_tok_off[s0], Tc = w.h_tok_off[s1] - t0;
+    CUDA_TRY(launch_embed_norm(w.tok_id + t0, Tc, m->embed, m->attn_norm, H, c.rms_eps, w.r, w.xn, st));
+    for (int l = 0; l < L; ++l) {
+      CUDA_TRY(launch_gemm(EPI_STORE_BF16, w.tm_xn, m->tm_qkv[l], Tc, m->qkv_dim, H, w.qkv, m->qkv_dim, w.err,
+                           m->num_sms, st));
+      CUDA_TRY(launch_qknorm_rope(w.qkv, Tc, m->qkv_dim, c.n_q_heads, c.n_kv_heads, m->q_norm + (size_t)l * HEAD_DIM,
+                                  m->k_norm + (size_t)l * HEAD_DIM, w.tok_pos + t0, m->rope, c.rms_eps, st));
+      AttnArgs aa{};
+      aa.items = w.items + plan.chunk_item[ci];
+      aa.n_items = plan.chunk_item[ci + 1] - plan.chunk_item[ci];
+      aa.tok_off = w.tok_off;
+      aa.tok0 = t0;
+      aa.qkv = w.qkv;
+      aa.ld_qkv = m->qkv_dim;
+      aa.out = w.o;
+      aa.ld_out = m->o_dim;
+      aa.slot_row = s->d_slot_row;
+      aa.layer = l;
+      aa.n_layers = L;
+      aa.Hq = c.n_q_heads;
+      aa.Hkv = c.n_kv_heads;
+      aa.mpad_cap = mpad;
+      aa.err = w.err;
+      CUDA_TRY(launch_attention(s->tm_pool, aa, st));
+      CUDA_TRY(launch_gemm(EPI_RESID_ADD_F32, w.tm_o, m->tm_o[l], Tc, H, m->o_dim, w.r, H, w.err, m->num_sms, st));
+      CUDA_TRY(launch_rmsnorm(w.r, Tc, H, m->mlp_norm + (size_t)l * H, c.rms_eps, w.xn, st));
+      CUDA_TRY(launch_gemm(EPI_SWIGLU_BF16, w.tm_xn, m->tm_gu[l], Tc, 2 * F, H, w.act, F, w.err, m->num_sms, st));
+      CUDA_TRY(launch_gemm(EPI_RESID_ADD_F32, w.tm_act, m->tm_down[l], Tc, H, F, w.r, H, w.err, m->num_sms, st));
+      if (l + 1 < L) CUDA_TRY(launch_rmsnorm(w.r, Tc, H, m->attn_norm + (size_t)(l + 1) * H, c.rms_eps, w.xn, st));
+    }
+    CUDA_TRY(launch_score(w.r, H, w.tok_off, t0, s0, s1, w.perm, m->final_norm, m->score_head, c.rms_eps, d_scores,
+                          st));
+  }
+  return DOPR_OK;
+}
+
+dopr_status check_ready(Model* m, Store* s) {
+  if (!m || !s) return fail(DOPR_ERR_INVALID_ARG, "model or store is NULL");
+  if (!same_shape(m->cfg, s->cfg)) return fail(DOPR_ERR_INVALID_ARG, "store shape does not match the model");
+  const int L = m->cfg.n_layers;
+  for (int k = 0; k < kind_count(); ++k)
+    for (int l = 0; l < (kind_is_global(k) ? 1 : L); ++l)
+      if (!m->have[k * L + l]) return fail(DOPR_ERR_INCOMPLETE, "weight kind %d layer %d was never put", k, l);
+  return DOPR_OK;
+}
+
+}  // namespace
+
+bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
+                       uint32_t box_cols, uint32_t box_rows, bool swizzle128) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {row_stride_bytes};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+}  // namespace dopr
+
+using namespace dopr;
+
+extern "C" {
+
+const char* dopr_version(void) { return "dopr-gb300 0.1 (sm_103a)"; }
+
+const char* dopr_last_error(void) { return g_last_error.c_str(); }
+
+int64_t dopr_prefix_bytes(const dopr_model_config* cfg, int32_t m) {
+  if (!cfg || m < 0 || cfg->n_layers <= 0 || cfg->n_kv_heads <= 0 || cfg->head_dim <= 0) return -1;
+  return (int64_t)m * cfg->n_layers * 2 * cfg->n_kv_heads * cfg->head_dim * 2;
+}
+
+dopr_status dopr_model_create(const dopr_model_config* cfg, dopr_model** out) {
+  g_last_error.clear();
+  if (!out) return fail(DOPR_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  STATUS_TRY(check_cfg(cfg));
+  if (!encode_fn()) return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable");
+  dopr_model* m = new dopr_model();
+  m->cfg = *cfg;
+  const auto& c = *cfg;
+  const size_t H = c.hidden, F = c.ffn, L = c.n_layers;
+  m->qkv_dim = (c.n_q_heads + 2 * c.n_kv_heads) * HEAD_DIM;
+  m->o_dim = c.n_q_heads * HEAD_DIM;
+  dopr_status st = DOPR_OK;
+  auto guard = [&](dopr_status s) {
+    if (s != DOPR_OK && st == DOPR_OK) st = s;
+    return s == DOPR_OK;
+  };
+  cudaGetDevice(&m->device);
+  cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
+  guard(gemm_setup() == cudaSuccess && attn_setup() == cudaSuccess
+            ? DOPR_OK
+            : fail(DOPR_ERR_CUDA, "kernel attribute setup failed: %s", cudaGetErrorString(cudaGetLastError())));
+  if (st == DOPR_OK &&
+      guard(dev_alloc(&m->embed, (size_t)c.vocab * H)) && guard(dev_alloc(&m->attn_norm, L * H)) &&
+      guard(dev_alloc(&m->w_qkv, L * m->qkv_dim * H)) && guard(dev_alloc(&m->q_norm, L * HEAD_DIM)) &&
+      guard(dev_alloc(&m->k_norm, L * HEAD_DIM)) && guard(dev_alloc(&m->w_o, L * H * m->o_dim)) &&
+      guard(dev_alloc(&m->mlp_norm, L * H)) && guard(dev_alloc(&m->w_gu, L * 2 * F * H)) &&
+      guard(dev_alloc(&m->w_down, L * H * F)) && guard(dev_alloc(&m->final_norm, H)) &&
+      guard(dev_alloc(&m->score_head, 2 * H)) && guard(dev_alloc(&m->rope, (size_t)c.max_position * (HEAD_DIM / 2)))) {
+    // RoPE table: angle = pos * theta^(-2i/128), evaluated in double on the host.
+    std::vector<float2> tab((size_t)c.max_position * (HEAD_DIM / 2));
+    for (int p = 0; p < c.max_position; ++p)
+      for (int i = 0; i < HEAD_DIM / 2; ++i) {
+        const double a = (double)p * pow((double)c.rope_theta, -2.0 * i / (double)HEAD_DIM);
+        tab[(size_t)p * (HEAD_DIM / 2) + i] = make_float2((float)cos(a), (float)sin(a));
+      }
+    if (cudaMemcpy(m->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice) != cudaSuccess)
+      guard(fail(DOPR_ERR_CUDA, "rope table upload failed"));
+  }
+  if (st == DOPR_OK) guard(build_weight_maps(m));
+  if (st == DOPR_OK) {
+    // Chunk size: enough rows to fill the GEMM tiles, bounded to ~2.5 GB of activations.
+    const int64_t per_tok = (int64_t)H * 6 + (int64_t)m->qkv_dim * 2 + (int64_t)m->o_dim * 2 + (int64_t)F * 2;
+    int64_t cap = (int64_t)2500 * 1000 * 1000 / per_tok;
+    cap = std::min<int64_t>(cap, 32768);
+    cap = std::max<int64_t>(cap, (int64_t)c.max_position);
+    cap = (cap + 127) / 128 * 128;
+    guard(alloc_chunk_buffers(m, (int)cap));
+  }
+  if (st != DOPR_OK) {
+    free_model(m);
+    delete m;
+    return st;
+  }
+  m->have.assign((size_t)kind_count() * L, 0);
+  *out = m;
+  return DOPR_OK;
+}
+
+dopr_status dopr_model_put_weight(dopr_model* m, int32_t kind, int32_t layer, const void* src, int64_t n_elems,
+                                  int32_t src_on_device) {
+  g_last_error.clear();
+  if (!m || !src) return fail(DOPR_ERR_INVALID_ARG, "model or src is NULL");
+  const auto& c = m->cfg;
+  const int64_t H = c.hidden, F = c.ffn, D = HEAD_DIM, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
+  if (kind < 0 || kind >= kind_count()) return fail(DOPR_ERR_INVALID_ARG, "bad weight kind %d", kind);
+  if (kind_is_global(kind)) layer = 0;
+  else if (layer < 0 || layer >= c.n_layers) return fail(DOPR_ERR_INVALID_ARG, "bad layer %d", layer);
+  const size_t l = (size_t)layer;
+  const cudaMemcpyKind dir = src_on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+  int64_t expect = 0;
+  bf16* dst = nullptr;
+  switch (kind) {
+    case DOPR_W_EMBED: expect = (int64_t)c.vocab * H; dst = m->embed; break;
+    case DOPR_W_ATTN_NORM: expect = H; dst = m->attn_norm + l * H; break;
+    case DOPR_W_Q: expect = Hq * D * H; dst = m->w_qkv + l * m->qkv_dim * H; break;
+    case DOPR_W_K: expect = Hkv * D * H; dst = m->w_qkv + (l * m->qkv_dim + Hq * D) * H; break;
+    case DOPR_W_V: expect = Hkv * D * H; dst = m->w_qkv + (l * m->qkv_dim + (Hq + Hkv) * D) * H; break;
+    case DOPR_W_Q_NORM: expect = D; dst = m->q_norm + l * D; break;
+    case DOPR_W_K_NORM: expect = D; dst = m->k_norm + l * D; break;
+    case DOPR_W_O: expect = H * Hq * D; dst = m->w_o + l * H * m->o_dim; break;
+    case DOPR_W_MLP_NORM: expect = H; dst = m->mlp_norm + l * H; break;
+    case DOPR_W_GATE:
+    case DOPR_W_UP: expect = F * H; dst = m->w_gu + l * 2 * F * H + (kind == DOPR_W_UP ? 128 * H : 0); break;
+    case DOPR_W_DOWN: expect = H * F; dst = m->w_down + l * H * F; break;
+    case DOPR_W_FINAL_NORM: expect = H; dst = m->final_norm; break;
+    case DOPR_W_SCORE_HEAD: expect = 2 * H; dst = m->score_head; break;
+  }
+  if (n_elems != expect)
+    return fail(DOPR_ERR_INVALID_ARG, "weight kind %d: %lld elements given, %lld expected", kind, (long long)n_elems,
+                (long long)expect);
+  CUDA_TRY(cudaSetDevice(m->device));
+  if (kind == DOPR_W_GATE || kind == DOPR_W_UP) {
+    // rows 128b..128b+127 of the source go to rows 256b (+128 for up) of the fused matrix
+    CUDA_TRY(cudaMemcpy2D(dst, 256 * H * 2, src, 128 * H * 2, 128 * H * 2, F / 128, dir));
+  } else {
+    CUDA_TRY(cudaMemcpy(dst, src, (size_t)expect * 2, dir));
+  }
+  m->have[(size_t)kind * c.n_layers + l] = 1;
+  return DOPR_OK;
+}
+
+dopr_status dopr_model_destroy(dopr_model* m) {
+  g_last_error.clear();
+  if (!m) return DOPR_OK;
+  cudaSetDevice(m->device);
+  free_model(m);
+  delete m;
+  return DOPR_OK;
+}
+
+dopr_status dopr_store_create(const dopr_model_config* cfg, int64_t max_doc_id, int64_t pool_bytes, dopr_store** out) {
+  g_last_error.clear();
+  if (!out) return fail(DOPR_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  STATUS_TRY(check_cfg(cfg));
+  if (max_doc_id < 0 || max_doc_id >= (1ll << 31) - 1) return fail(DOPR_ERR_INVALID_ARG, "bad max_doc_id");
+  if (pool_bytes < 0) return fail(DOPR_ERR_INVALID_ARG, "bad pool_bytes");
+  if (pool_bytes / 256 >= (1ll << 31)) return fail(DOPR_ERR_UNSUPPORTED, "pool above 512 GiB");
+  dopr_store* s = new dopr_store();
+  s->cfg = *cfg;
+  s->max_doc_id = max_doc_id;
+  s->pool_rows = pool_bytes / 256;
+  s->pool_bytes = s->pool_rows * 256;
+  cudaGetDevice(&s->device);
+  const size_t nd = (size_t)max_doc_id + 1;
+  dopr_status st = DOPR_OK;
+  auto guard = [&](dopr_status x) {
+    if (x != DOPR_OK && st == DOPR_OK) st = x;
+    return x == DOPR_OK;
+  };
+  if (guard(dev_alloc(&s->pool, (size_t)std::max<int64_t>(s->pool_bytes, 256))) &&
+      guard(dev_alloc(&s->d_slot_of, nd)) && guard(dev_alloc(&s->d_slot_m, nd)) &&
+      guard(dev_alloc(&s->d_slot_row, nd)) && guard(dev_alloc(&s->d_slot_ok, nd))) {
+    if (cudaMemset(s->d_slot_of, 0xFF, nd * sizeof(int32_t)) != cudaSuccess ||
+        cudaMemset(s->d_slot_ok, 0, nd) != cudaSuccess || cudaMemset(s->d_slot_m, 0, nd * sizeof(int32_t)) ||
+        cudaMemset(s->pool, 0, (size_t)std::max<int64_t>(s->pool_bytes, 256)) != cudaSuccess)
+      guard(fail(DOPR_ERR_CUDA, "store initialisation failed"));
+  }
+  if (st == DOPR_OK &&
+      !make_tmap_bf16_2d(&s->tm_pool, s->pool, HEAD_DIM, std::max<int64_t>(s->pool_rows, 1), HEAD_DIM * 2, 64, 64, true))
+    guard(fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for the store pool"));
+  if (st != DOPR_OK) {
+    free_store(s);
+    delete s;
+    return st;
+  }
+  s->tm_pool_ok = true;
+  s->slot_of.assign(nd, -1);
+  *out = s;
+  return DOPR_OK;
+}
+
+dopr_status dopr_store_put(dopr_store* s, int64_t doc_id, int32_t m, int32_t layer, const void* k, const void* v,
+                           int32_t src_on_device) {
+  g_last_error.clear();
+  if (!s) return fail(DOPR_ERR_INVALID_ARG, "store is NULL");
+  const auto& c = s->cfg;
+  if (doc_id < 0 || doc_id > s->max_doc_id) return fail(DOPR_ERR_INVALID_ARG, "doc_id %lld out of range", (long long)doc_id);
+  if (m < 0 || m > MAX_PREFIX) return fail(DOPR_ERR_INVALID_ARG, "m = %d outside [0, %d]", m, MAX_PREFIX);
+  if (layer < 0 || layer >= c.n_layers) return fail(DOPR_ERR_INVALID_ARG, "bad layer %d", layer);
+  if (m > 0 && (!k || !v)) return fail(DOPR_ERR_INVALID_ARG, "k or v is NULL");
+  int32_t slot = s->slot_of[doc_id];
+  if (slot >= 0 && s->slot_m[slot] != m)
+    return fail(DOPR_ERR_INVALID_ARG, "doc %lld was stored with m = %d, not %d", (long long)doc_id, s->slot_m[slot], m);
+  const int64_t Hkv = c.n_kv_heads;
+  const int64_t rows_per_layer = 2 * Hkv * m;  // K and V, [head][m] rows of 128
+  CUDA_TRY(cudaSetDevice(s->device));
+  if (slot < 0) {
+    const int64_t need = rows_per_layer * c.n_layers;
+    if (s->used_rows + need > s->pool_rows)
+      return fail(DOPR_ERR_OUT_OF_MEMORY, "store pool full (%lld of %lld rows used, %lld needed)",
+                  (long long)s->used_rows, (long long)s->pool_rows, (long long)need);
+    slot = s->n_slots++;
+    s->slot_m.push_back(m);
+    s->slot_row.push_back(s->used_rows);
+    s->slot_layers.emplace_back(c.n_layers, 0);
+    s->slot_ok.push_back(0);
+    s->used_rows += need;
+    s->slot_of[doc_id] = slot;
+    const int64_t row = s->slot_row[slot];
+    CUDA_TRY(cudaMemcpy(s->d_slot_m + slot, &m, sizeof(int32_t), cudaMemcpyHostToDevice));
+    CUDA_TRY(cudaMemcpy(s->d_slot_row + slot, &row, sizeof(int64_t), cudaMemcpyHostToDevice));
+    CUDA_TRY(cudaMemcpy(s->d_slot_of + doc_id, &slot, sizeof(int32_t), cudaMemcpyHostToDevice));
+    s->max_m = std::max(s->max_m, m);
+  }
+  if (m > 0) {
+    const size_t bytes = (size_t)m * Hkv * HEAD_DIM * 2;
+    bf16* base = reinterpret_cast<bf16*>(s->pool) + (size_t)(s->slot_row[slot] + layer * rows_per_layer) * HEAD_DIM;
+    const bf16 *dk = static_cast<const bf16*>(k), *dv = static_cast<const bf16*>(v);
+    bf16* stage = nullptr;
+    if (!src_on_device) {
+      CUDA_TRY(cudaMalloc(&stage, 2 * bytes));
+      cudaError_t e1 = cudaMemcpy(stage, k, bytes, cudaMemcpyHostToDevice);
+      cudaError_t e2 = cudaMemcpy(stage + bytes / 2, v, bytes, cudaMemcpyHostToDevice);
+      if (e1 != cudaSuccess || e2 != cudaSuccess) {
+        cudaFree(stage);
+        return fail(DOPR_ERR_CUDA, "prefix upload failed");
+      }
+      dk = stage;
+      dv = stage + bytes / 2;
+    }
+    cudaError_t e = launch_store_transpose(dk, dv, m, (int)Hkv, base, base + (size_t)Hkv * m * HEAD_DIM, 0);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(0);
+    if (stage) cudaFree(stage);
+    if (e != cudaSuccess) return fail(DOPR_ERR_CUDA, "prefix store copy failed: %s", cudaGetErrorString(e));
+  }
+  if (!s->slot_layers[slot][layer]) {
+    s->slot_layers[slot][layer] = 1;
+    bool all = true;
+    for (int l = 0; l < c.n_layers; ++l) all = all && s->slot_layers[slot][l];
+    if (all) {
+      s->slot_ok[slot] = 1;
+      const uint8_t one = 1;
+      CUDA_TRY(cudaMemcpy(s->d_slot_ok + slot, &one, 1, cudaMemcpyHostToDevice));
+    }
+  }
+  return DOPR_OK;
+}
+
+dopr_status dopr_store_destroy(dopr_store* s) {
+  g_last_error.clear();
+  if (!s) return DOPR_OK;
+  cudaSetDevice(s->device);
+  free_store(s);
+  delete s;
+  return DOPR_OK;
+}
+
+dopr_status dopr_score(dopr_model* m, dopr_store* s, int32_t n, const int32_t* q_offsets, const int32_t* q_tokens,
+                       const int64_t* doc_ids, float* scores, void* cuda_stream, int32_t io_on_device) {
+  g_last_error.clear();
+  STATUS_TRY(check_ready(m, s));
+  if (n < 0) return fail(DOPR_ERR_INVALID_ARG, "n_pairs < 0");
+  if (n == 0) return DOPR_OK;
+  if (!q_offsets || !doc_ids || !scores) return fail(DOPR_ERR_INVALID_ARG, "NULL array");
+  CUDA_TRY(cudaSetDevice(m->device));
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  Workspace& w = m->ws;
+  const int32_t *dqo = q_offsets, *dqt = q_tokens;
+  const int64_t* ddoc = doc_ids;
+  float* dsc = scores;
+  if (!io_on_device) {
+    if (n > 0 && q_offsets[n] > 0 && !q_tokens) return fail(DOPR_ERR_INVALID_ARG, "q_tokens is NULL");
+    STATUS_TRY(validate_host_inputs(m, s, n, q_offsets, q_tokens, doc_ids));
+    const int64_t nq = q_offsets[n];
+    STATUS_TRY(ensure_call_buffers(m, n, 0, std::max<int64_t>(nq, 1), s->max_doc_id + 1));
+    CUDA_TRY(cudaMemcpyAsync(w.q_off, q_offsets, sizeof(int32_t) * (n + 1), cudaMemcpyHostToDevice, st));
+    if (nq > 0) CUDA_TRY(cudaMemcpyAsync(w.q_tok, q_tokens, sizeof(int32_t) * nq, cudaMemcpyHostToDevice, st));
+    CUDA_TRY(cudaMemcpyAsync(w.doc_ids, doc_ids, sizeof(int64_t) * n, cudaMemcpyHostToDevice, st));
+    dqo = w.q_off;
+    dqt = w.q_tok;
+    ddoc = w.doc_ids;
+    dsc = w.scores;
+  } else {
+    STATUS_TRY(ensure_call_buffers(m, n, 0, 0, s->max_doc_id + 1));
+  }
+  Plan plan;
+  STATUS_TRY(run_packer(m, s, n, dqo, dqt, ddoc, st, plan));
+  STATUS_TRY(run_layers(m, s, plan, dsc, st));
+  if (!io_on_device) CUDA_TRY(cudaMemcpyAsync(scores, w.scores, sizeof(float) * n, cudaMemcpyDeviceToHost, st));
+  CUDA_TRY(cudaMemcpyAsync(w.h_err, w.err, sizeof(int), cudaMemcpyDeviceToHost, st));
+  CUDA_TRY(cudaStreamSynchronize(st));
+  return map_device_error(*w.h_err);
+}
+
+dopr_status dopr_debug_pack_plan(dopr_model* m, dopr_store* s, int32_t n, const int32_t* q_offsets,
+                                 const int32_t* q_tokens, const int64_t* doc_ids, int32_t* perm, int32_t* tok_off,
+                                 int32_t* tok_pos, int32_t* tok_id, int32_t* tok_pair) {
+  g_last_error.clear();
+  if (!m || !s) return fail(DOPR_ERR_INVALID_ARG, "model or store is NULL");
+  if (!same_shape(m->cfg, s->cfg)) return fail(DOPR_ERR_INVALID_ARG, "store shape does not match the model");
+  if (n < 0 || !q_offsets || (n > 0 && (!doc_ids || !perm || !tok_off))) return fail(DOPR_ERR_INVALID_ARG, "bad args");
+  if (n == 0) {
+    tok_off[0] = 0;
+    return DOPR_OK;
+  }
+  STATUS_TRY(validate_host_inputs(m, s, n, q_offsets, q_tokens, doc_ids));
+  CUDA_TRY(cudaSetDevice(m->device));
+  Workspace& w = m->ws;
+  const int64_t nq = q_offsets[n];
+  STATUS_TRY(ensure_call_buffers(m, n, 0, std::max<int64_t>(nq, 1), s->max_doc_id + 1));
+  cudaStream_t st = 0;
+  CUDA_TRY(cudaMemcpy(w.q_off, q_offsets, sizeof(int32_t) * (n + 1), cudaMemcpyHostToDevice));
+  if (nq > 0) CUDA_TRY(cudaMemcpy(w.q_tok, q_tokens, sizeof(int32_t) * nq, cudaMemcpyHostToDevice));
+  CUDA_TRY(cudaMemcpy(w.doc_ids, doc_ids, sizeof(int64_t) * n, cudaMemcpyHostToDevice));
+  Plan plan;
+  STATUS_TRY(run_packer(m, s, n, w.q_off, w.q_tok, w.doc_ids, st, plan));
+  const int64_t T = plan.n_tokens;
+  CUDA_TRY(cudaStreamSynchronize(st));
+  CUDA_TRY(cudaMemcpy(perm, w.perm, sizeof(int32_t) * n, cudaMemcpyDeviceToHost));
+  CUDA_TRY(cudaMemcpy(tok_off, w.tok_off, sizeof(int32_t) * (n + 1), cudaMemcpyDeviceToHost));
+  if (tok_pos) CUDA_TRY(cudaMemcpy(tok_pos, w.tok_pos, sizeof(int32_t) * T, cudaMemcpyDeviceToHost));
+  if (tok_id) CUDA_TRY(cudaMemcpy(tok_id, w.tok_id, sizeof(int32_t) * T, cudaMemcpyDeviceToHost));
+  if (tok_pair) CUDA_TRY(cudaMemcpy(tok_pair, w.tok_pair, sizeof(int32_t) * T, cudaMemcpyDeviceToHost));
+  CUDA_TRY(cudaMemcpy(w.h_err, w.err, sizeof(int), cudaMemcpyDeviceToHost));
+  return map_device_error(*w.h_err);
+}
+
+dopr_status dopr_debug_gemm(int32_t M, int32_t N, int32_t K, const void* A, const void* B, void* out,
+                            int32_t epilogue, void* cuda_stream) {
+  g_last_error.clear();
+  if (M < 0 || N <= 0 || K <= 0 || !A || !B || !out) return fail(DOPR_ERR_INVALID_ARG, "bad gemm args");
+  if (K % GEMM_BK || N % GEMM_BN) return fail(DOPR_ERR_UNSUPPORTED, "K % 64 and N % 256 must be 0");
+  if (epilogue < 0 || epilogue > 2) return fail(DOPR_ERR_INVALID_ARG, "bad epilogue %d", epilogue);
+  if (M == 0) return DOPR_OK;
+  if (gemm_setup() != cudaSuccess) return fail(DOPR_ERR_CUDA, "gemm setup failed");
+  CUtensorMap ta, tb;
+  if (!make_tmap_bf16_2d(&ta, A, K, M, (uint64_t)K * 2, GEMM_BK, GEMM_BM, true) ||
+      !make_tmap_bf16_2d(&tb, B, K, N, (uint64_t)K * 2, GEMM_BK, GEMM_BN, true))
+    return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed (pointers must be 16-byte aligned)");
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  int* err = nullptr;
+  CUDA_TRY(cudaMalloc(&err, sizeof(int)));
+  cudaMemsetAsync(err, 0, sizeof(int), st);
+  const int64_t ld = epilogue == EPI_SWIGLU_BF16 ? N / 2 : N;
+  cudaError_t e = launch_gemm(epilogue, ta, tb, M, N, K, out, ld, err, sms, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  int h = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&h, err, sizeof(int), cudaMemcpyDeviceToHost);
+  cudaFree(err);
+  if (e != cudaSuccess) return fail(DOPR_ERR_CUDA, "gemm failed: %s", cudaGetErrorString(e));
+  return map_device_error(h);
+}
+
+dopr_status dopr_debug_wait_timeout(int32_t timeout_ms) {
+  g_last_error.clear();
+  if (timeout_ms <= 0 || timeout_ms > 10000) return fail(DOPR_ERR_INVALID_ARG, "timeout_ms in (0, 10000]");
+  int* err = nullptr;
+  CUDA_TRY(cudaMalloc(&err, sizeof(int)));
+  cudaMemset(err, 0, sizeof(int));
+  cudaError_t e = launch_wait_timeout_probe(err, (uint64_t)timeout_ms * 1000000ull, 0);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  int h = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&h, err, sizeof(int), cudaMemcpyDeviceToHost);
+  cudaFree(err);
+  if (e != cudaSuccess) return fail(DOPR_ERR_CUDA, "probe failed: %s", cudaGetErrorString(e));
+  return map_device_error(h);
+}
+
+}  // extern "C"

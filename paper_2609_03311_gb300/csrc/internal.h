@@ -1,0 +1,181 @@
+// internal.h -- host-side structures of libdopr and the launchers each kernel
+// file exports to the engine (abi.cu).  Not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/dopr.h"
+
+namespace dopr {
+
+typedef __nv_bfloat16 bf16;
+
+constexpr int HEAD_DIM = 128;
+constexpr int MAX_PREFIX = 256;       // largest m the store accepts
+constexpr int ATTN_MAX_PAIRS = 8;     // pairs of one doc per attention work item
+constexpr uint64_t WAIT_TIMEOUT_NS = 4000000000ull;  // bounded device waits: 4 s
+
+// One attention work item: consecutive sorted pairs that share a document.
+struct AttnItem {
+  int32_t pair_begin, pair_end;  // sorted pair indices [begin, end)
+  int32_t slot;                  // store slot of the document
+  int32_t m;                     // its prefix length
+};
+
+struct Store {
+  dopr_model_config cfg{};
+  int device = 0;
+  int64_t max_doc_id = 0;
+  int64_t pool_bytes = 0, pool_rows = 0, used_rows = 0;  // rows of 128 bf16 (256 B)
+  uint8_t* pool = nullptr;
+  int32_t* d_slot_of = nullptr;     // [max_doc_id+1] doc -> slot, -1 absent
+  int32_t* d_slot_m = nullptr;      // [max_doc_id+1] per slot prefix length
+  int64_t* d_slot_row = nullptr;    // [max_doc_id+1] first pool row of the slot block
+  uint8_t* d_slot_ok = nullptr;     // [max_doc_id+1] all layers present
+  std::vector<int32_t> slot_of;     // host mirrors
+  std::vector<int32_t> slot_m;
+  std::vector<int64_t> slot_row;
+  std::vector<std::vector<uint8_t>> slot_layers;
+  std::vector<uint8_t> slot_ok;
+  int32_t n_slots = 0;
+  int32_t max_m = 0;
+  CUtensorMap tm_pool{};
+  bool tm_pool_ok = false;
+};
+
+struct Workspace {
+  int chunk_cap = 0;  // tokens per chunk
+  float* r = nullptr;          // [chunk][H] fp32 residual stream
+  bf16* xn = nullptr;          // [chunk][H] normed activations
+  bf16* qkv = nullptr;         // [chunk][(Hq+2Hkv)*128]
+  bf16* o = nullptr;           // [chunk][Hq*128]
+  bf16* act = nullptr;         // [chunk][F]
+  CUtensorMap tm_xn{}, tm_o{}, tm_act{};
+  // per call, grown on demand
+  int64_t pair_cap = 0, tok_cap = 0, qtok_cap = 0, doc_cap = 0, item_cap = 0;
+  int32_t* q_off = nullptr;
+  int32_t* q_tok = nullptr;
+  int64_t* doc_ids = nullptr;
+  float* scores = nullptr;
+  int32_t* pair_slot = nullptr;
+  int32_t* perm = nullptr;
+  int32_t* sorted_slot = nullptr;
+  int32_t* tok_off = nullptr;
+  int32_t* tok_id = nullptr;
+  int32_t* tok_pos = nullptr;
+  int32_t* tok_pair = nullptr;
+  int32_t* doc_count = nullptr;  // [max_doc_id+1] counting-sort buckets
+  AttnItem* items = nullptr;
+  int* err = nullptr;
+  // pinned host staging
+  int32_t* h_tok_off = nullptr;
+  int32_t* h_sorted_slot = nullptr;
+  int* h_err = nullptr;
+  AttnItem* h_items = nullptr;
+  int64_t h_pair_cap = 0, h_item_cap = 0;
+};
+
+struct Model {
+  dopr_model_config cfg{};
+  int device = 0;
+  int num_sms = 0;
+  int qkv_dim = 0;  // (Hq + 2 Hkv) * 128
+  int o_dim = 0;    // Hq * 128
+  bf16* embed = nullptr;       // [V][H]
+  bf16* attn_norm = nullptr;   // [L][H]
+  bf16* w_qkv = nullptr;       // [L][qkv_dim][H]
+  bf16* q_norm = nullptr;      // [L][128]
+  bf16* k_norm = nullptr;      // [L][128]
+  bf16* w_o = nullptr;         // [L][H][o_dim]
+  bf16* mlp_norm = nullptr;    // [L][H]
+  bf16* w_gu = nullptr;        // [L][2F][H], gate/up interleaved in 128-row blocks
+  bf16* w_down = nullptr;      // [L][H][F]
+  bf16* final_norm = nullptr;  // [H]
+  bf16* score_head = nullptr;  // [2][H]
+  float2* rope = nullptr;      // [max_position][64] (cos, sin)
+  std::vector<uint8_t> have;   // [kind * L + layer]
+  std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
+  bool maps_ok = false;
+  Workspace ws;
+};
+
+// ------------------------------------------------------------ launchers
+// Tensor map helper (driver entry point resolved at run time).
+bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
+                       uint32_t box_cols, uint32_t box_rows, bool swizzle128);
+
+// GEMM epilogues.
+enum GemmEpi : int { EPI_STORE_BF16 = 0, EPI_RESID_ADD_F32 = 1, EPI_SWIGLU_BF16 = 2 };
+constexpr int GEMM_BM = 128, GEMM_BN = 256, GEMM_BK = 64;
+cudaError_t gemm_setup();
+// C[M][N] = A[M][K] * B[N][K]^T with the given epilogue writing `out` (ld in elements).
+cudaError_t launch_gemm(int epi, const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
+                        int64_t ld_out, int* err, int num_sms, cudaStream_t st);
+
+// Row kernels.
+cudaError_t launch_embed_norm(const int32_t* tok_id, int T, const bf16* embed, const bf16* gain, int H, float eps,
+                              float* r, bf16* xn, cudaStream_t st);
+cudaError_t launch_rmsnorm(const float* r, int T, int H, const bf16* gain, float eps, bf16* xn, cudaStream_t st);
+cudaError_t launch_qknorm_rope(bf16* qkv, int T, int ld, int Hq, int Hkv, const bf16* qn, const bf16* kn,
+                               const int32_t* tok_pos, const float2* rope, float eps, cudaStream_t st);
+cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end,
+                         const int32_t* perm, const bf16* gain, const bf16* head, float eps, float* scores,
+                         cudaStream_t st);
+cudaError_t launch_store_transpose(const bf16* k, const bf16* v, int m, int Hkv, bf16* dk, bf16* dv,
+                                   cudaStream_t st);
+
+// Attention.
+struct AttnArgs {
+  const AttnItem* items;
+  int n_items;
+  const int32_t* tok_off;  // sorted pair -> first packed token
+  int32_t tok0;            // first packed token of this chunk
+  const bf16* qkv;
+  int ld_qkv;
+  bf16* out;
+  int ld_out;
+  const int64_t* slot_row;
+  int layer, n_layers, Hq, Hkv;
+  int mpad_cap;  // prefix rows reserved in shared memory (multiple of 64)
+  int* err;
+};
+cudaError_t attn_setup();
+cudaError_t launch_attention(const CUtensorMap& tm_pool, const AttnArgs& a, cudaStream_t st);
+
+// Packer.
+struct PackArgs {
+  int n_pairs;
+  const int32_t* q_off;
+  const int32_t* q_tok;
+  const int64_t* doc_ids;
+  int64_t max_doc_id;
+  const int32_t* slot_of;
+  const int32_t* slot_m;
+  const uint8_t* slot_ok;
+  int vocab, score_token, max_position;
+  int32_t* doc_count;  // [max_doc_id+1], zeroed by the launcher
+  int32_t* pair_slot;
+  int32_t* perm;
+  int32_t* sorted_slot;
+  int32_t* tok_off;
+  int32_t* tok_id;
+  int32_t* tok_pos;
+  int32_t* tok_pair;
+  int* err;
+};
+// Device packer, first part: validation, stable sort by doc id, packed token
+// offsets (tok_off).  Zeroes doc_count itself.
+cudaError_t launch_pack_order(const PackArgs& a, cudaStream_t st);
+// Second part, once the token buffers are sized: token ids, positions, pair index.
+cudaError_t launch_pack_tokens(const PackArgs& a, cudaStream_t st);
+
+// Debug kernel: bounded wait on a barrier nothing completes.
+cudaError_t launch_wait_timeout_probe(int* err, uint64_t timeout_ns, cudaStream_t st);
+
+}  // namespace dopr
