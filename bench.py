@@ -1,0 +1,459 @@
+#!/usr/bin/env python
+"""Benchmark of the DoPR online scoring pass on GB300.
+
+One step = one dopr_score call over one batch of the workload: Q queries'
+candidate lists (default 20 queries x 100 candidates = 2,000 pairs of the
+Qwen3-8B, m = 64, Zipf(1.1) workload).  Steps walk through the workload's
+200 queries; with --gpus N every rank scores its own batches (pairs are
+independent: weak scaling, no data-path collective).
+
+Printed JSON line (rank 0):
+  value      scored pairs/s, inputs resident in HBM (io_on_device = 1), max over ranks
+  e2e        same metric through the C ABI with pinned host buffers (H2D of the
+             batch and D2H of its scores inside the timed region)
+  roofline   dominant kernel (the tcgen05 projection GEMM family): algorithmic
+             FLOPs / CUDA-event time of its launches in the timed region, vs
+             the measured sustained bf16 peak
+  kernels    the same accounting for every kernel family
+  cpu_baseline  the fp64 oracle timed on a bounded sample on the host cores
+  --impl reference  times the oracle alone (the reference arm of this workload)
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "scored query-doc pairs/sec at 1 GB300 (Qwen3-8B shape, m=64); p50 batch latency"
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["dopr", "reference"], default="dopr")
+    ap.add_argument("--workload", default="qwen3-8b-m64")
+    ap.add_argument("--queries-per-step", type=int, default=20)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0, help="bound of the oracle CPU-baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--latency-queries", type=int, default=10)
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        p = json.load(open(path))
+        return {"hbm_gbs": p["hbm_gbs"], "bf16_tflops": p["bf16_tflops"],
+                "bf16_tflops_sustained": p.get("bf16_tflops_sustained", p["bf16_tflops"]), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+    FIELDS = "index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown," \
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown," \
+             "clocks_event_reasons.sw_power_cap"
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.lines = []
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# -------------------------------------------------------------- workload
+
+def build_pairs(wl, seed):
+    from paper_2609_03311_gb300 import synth
+
+    pairs = synth.make_workload_pairs(wl, seed=seed)
+    if wl.fulldoc_tokens:
+        # uncompressed pointwise scoring: [doc tokens ; query] per pair, no prefix
+        qo, qt, docs = pairs["q_offsets"], pairs["q_tokens"], pairs["doc_ids"]
+        cache = {}
+        seqs = []
+        for p in range(len(docs)):
+            d = int(docs[p])
+            if d not in cache:
+                cache[d] = synth.make_fulldoc_tokens(wl, d, seed=seed)
+            seqs.append(np.concatenate([cache[d], qt[qo[p]:qo[p + 1]]]))
+        pairs["q_offsets"] = np.concatenate([[0], np.cumsum([len(s) for s in seqs])]).astype(np.int32)
+        pairs["q_tokens"] = np.concatenate(seqs).astype(np.int32)
+    return pairs
+
+
+def slice_pairs(pairs, p0, p1):
+    qo = pairs["q_offsets"]
+    return {"q_offsets": (qo[p0:p1 + 1] - qo[p0]).astype(np.int32),
+            "q_tokens": pairs["q_tokens"][qo[p0]:qo[p1]].astype(np.int32),
+            "doc_ids": pairs["doc_ids"][p0:p1].astype(np.int64)}
+
+
+def oracle_sample(wl, w_host, doc_m, pairs, idx, seed, deadline_s, gen_device):
+    """Score pairs idx[0], idx[1], ... with the oracle until deadline_s of CPU
+    time is used (at least one pair).  Returns (scores dict, seconds, threads)."""
+    import oracle
+    from paper_2609_03311_gb300 import synth
+
+    s = wl.model
+    om = oracle.OracleModel(oracle.Shape(s.n_layers, s.hidden, s.n_q_heads, s.n_kv_heads, s.head_dim, s.ffn,
+                                         s.vocab, s.rope_theta, s.rms_eps, s.score_token_id), w_host)
+    got = {}
+    t0 = time.perf_counter()
+    for p in idx:
+        d = int(pairs["doc_ids"][p])
+        m = int(doc_m[d])
+        # the same draw the store received (same seed, same generator device)
+        k, v = synth.make_prefix(s, m, d, seed=seed, device=gen_device)
+        one = slice_pairs(pairs, p, p + 1)
+        got[int(p)] = float(om.score_pairs(one["q_offsets"], one["q_tokens"], [0], [(k.cpu(), v.cpu())])[0])
+        if time.perf_counter() - t0 >= deadline_s:
+            break
+    return got, time.perf_counter() - t0, oracle.num_threads()
+
+
+def setup(wl, seed, device, need_host_weights):
+    """Random-init model and prefix store on `device`; optional host copy of
+    the weights for the oracle."""
+    import torch
+
+    from paper_2609_03311_gb300 import dopr, synth
+
+    s = wl.model
+    w = synth.make_weights(s, seed=seed, device=device, norms="ones")
+    max_pos = max(wl.m_choices) + wl.fulldoc_tokens + wl.qlen_max + 2
+    cfg = dopr.make_config(s, max_position=max(1024, max_pos))
+    model = dopr.Model(cfg, w)
+    w_host = None
+    if need_host_weights:
+        w_host = {k: (v.cpu() if isinstance(v, torch.Tensor) else [t.cpu() for t in v]) for k, v in w.items()}
+    del w
+    torch.cuda.empty_cache()
+    doc_m = synth.doc_prefix_lengths(wl, seed=seed)
+    pool = sum(dopr.prefix_bytes(cfg, int(m)) for m in doc_m) + (1 << 20)
+    store = dopr.Store(cfg, wl.n_docs - 1, pool)
+    for d in range(wl.n_docs):
+        k, v = synth.make_prefix(s, int(doc_m[d]), d, seed=seed, device=device)
+        store.put(d, k, v)
+    torch.cuda.synchronize()
+    return cfg, model, store, doc_m, w_host
+
+
+def gemm_traffic_record():
+    """ncu-measured DRAM traffic per GEMM launch, valid only for the kernel
+    source it was captured from (else None)."""
+    path = os.path.join(ROOT, "profiles", "gemm_traffic.json")
+    if not os.path.exists(path):
+        return None
+    rec = json.load(open(path))
+    src = open(os.path.join(ROOT, "paper_2609_03311_gb300", "csrc", "k_gemm.cu"), "rb").read()
+    if rec.get("k_gemm_sha256") != hashlib.sha256(src).hexdigest():
+        return None
+    return rec
+
+
+# ------------------------------------------------------------------ arms
+
+def run_dopr(args, rank, world, local_rank, dist):
+    import torch
+
+    from paper_2609_03311_gb300 import dopr, synth
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    wl = synth.WORKLOADS[args.workload]
+    want_cpu = (not args.no_cpu_baseline) and rank == 0 and world == 1
+    cfg, model, store, doc_m, w_host = setup(wl, args.seed, dev, want_cpu)
+    pairs = build_pairs(wl, args.seed)
+    per_q = wl.docs_per_query
+    Q = max(1, min(args.queries_per_step, wl.n_queries))
+    n_batches = wl.n_queries // Q
+    batches = []
+    for b in range(n_batches):
+        sl = slice_pairs(pairs, b * Q * per_q, (b + 1) * Q * per_q)
+        sl["dev"] = (torch.tensor(sl["q_offsets"], device=dev), torch.tensor(sl["q_tokens"], device=dev),
+                     torch.tensor(sl["doc_ids"], device=dev))
+        sl["pin"] = (torch.tensor(sl["q_offsets"]).pin_memory(), torch.tensor(sl["q_tokens"]).pin_memory(),
+                     torch.tensor(sl["doc_ids"]).pin_memory())
+        sl["first_pair"] = b * Q * per_q
+        batches.append(sl)
+    stream = torch.cuda.current_stream(dev)
+
+    def batch_for(step):
+        return batches[(rank + step * world) % n_batches]
+
+    def step_dev(b):
+        qo, qt, di = b["dev"]
+        return dopr.score(model, store, qo, qt, di)
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    def max_over_ranks(x):
+        if dist is None:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev if dist.get_backend() == "nccl" else "cpu")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def sum_over_ranks(x):
+        if dist is None:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev if dist.get_backend() == "nccl" else "cpu")
+        dist.all_reduce(t, op=dist.ReduceOp.SUM)
+        return float(t.item())
+
+    for i in range(args.warmup):
+        step_dev(batch_for(i))
+    torch.cuda.synchronize()
+
+    # ---------------- timed region: device-resident inputs
+    dopr.profile_enable(model, True)
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    ev[0].record(stream)
+    pairs_done = 0
+    outs = []
+    for i in range(args.steps):
+        b = batch_for(args.warmup + i)
+        outs.append((b, step_dev(b)))
+        ev[i + 1].record(stream)
+        pairs_done += len(b["doc_ids"])
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    prof = dopr.profile_read(model)
+    dopr.profile_enable(model, False)
+    step_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)]
+    total_ms = max_over_ranks(ev[0].elapsed_time(ev[-1]))
+    all_pairs = sum_over_ranks(pairs_done)
+    value = all_pairs / (total_ms / 1e3)
+
+    # ---------------- e2e: pinned host buffers through the C ABI
+    e2e = None
+    if not args.no_e2e:
+        out_pin = torch.empty(Q * per_q, dtype=torch.float32).pin_memory()
+        barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        h2d = d2h = 0
+        for i in range(args.steps):
+            b = batch_for(args.warmup + i)
+            qo, qt, di = b["pin"]
+            n = len(b["doc_ids"])
+            dopr.score(model, store, qo, qt, di, out=out_pin[:n])
+            h2d += qo.numel() * 4 + qt.numel() * 4 + di.numel() * 8
+            d2h += n * 4
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        e_ms = max_over_ranks(e0.elapsed_time(e1))
+        e2e = {"value": all_pairs / (e_ms / 1e3), "unit": "pairs/s", "h2d_bytes_per_step": h2d // args.steps,
+               "d2h_bytes_per_step": d2h // args.steps}
+
+    # ---------------- per-query latency (one call per query's candidate list)
+    lat = []
+    for qi in range(min(args.latency_queries, wl.n_queries)):
+        sl = slice_pairs(pairs, qi * per_q, (qi + 1) * per_q)
+        qo, qt, di = (torch.tensor(sl["q_offsets"], device=dev), torch.tensor(sl["q_tokens"], device=dev),
+                      torch.tensor(sl["doc_ids"], device=dev))
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        dopr.score(model, store, qo, qt, di)
+        torch.cuda.synchronize()
+        lat.append((time.perf_counter() - t0) * 1e3)
+    lat_sorted = sorted(lat[1:] if len(lat) > 1 else lat)
+
+    # ---------------- roofline accounting from the live CUDA-event timing
+    peaks = measured_peaks()
+    gemm_fams = ["gemm_qkv", "gemm_o", "gemm_gate_up", "gemm_down"]
+    tot_ms = sum(v["time_ms"] for v in prof.values()) or 1e-9
+    g_ms = sum(prof[f]["time_ms"] for f in gemm_fams)
+    g_flops = sum(prof[f]["flops"] for f in gemm_fams)
+    g_launch = sum(prof[f]["launches"] for f in gemm_fams)
+    g_bytes = sum(prof[f]["bytes"] for f in gemm_fams)
+    achieved = g_flops / (g_ms / 1e3) / 1e12 if g_ms > 0 else None
+    traffic = gemm_traffic_record()
+    roofline = {"bound": "tensor", "kernel": "k_gemm_tc (QKV/O/gate-up/down projections)",
+                "achieved": achieved, "peak": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s",
+                "frac": (achieved / peaks["bf16_tflops_sustained"]) if achieved else None,
+                "peak_source": f"{peaks['source']} sustained bf16 (kernel timed inside a long step)",
+                "traffic": (traffic["dram_bytes_per_launch"] if traffic else None),
+                "algorithmic_flops_per_launch": g_flops / max(g_launch, 1),
+                "algorithmic_bytes_per_launch": g_bytes / max(g_launch, 1),
+                "share_of_step": g_ms / tot_ms}
+    kernels = {}
+    for name, v in prof.items():
+        if v["launches"] == 0:
+            continue
+        t_s = v["time_ms"] / 1e3
+        ent = {"launches_per_step": v["launches"] / args.steps, "ms_per_step": v["time_ms"] / args.steps,
+               "share": v["time_ms"] / tot_ms}
+        if t_s > 0:
+            tf = v["flops"] / t_s / 1e12
+            gbs = v["bytes"] / t_s / 1e9
+            t_roof = max(v["flops"] / (peaks["bf16_tflops_sustained"] * 1e12), v["bytes"] / (peaks["hbm_gbs"] * 1e9))
+            ent.update({"tflops": tf, "gbs": gbs, "roofline_frac": t_roof / t_s})
+        kernels[name] = ent
+    gpu_launches = sum(v["launches"] for v in prof.values())
+
+    # ---------------- CPU baseline: the oracle on a bounded sample, rank 0, N = 1
+    cpu = parity = None
+    if want_cpu:
+        b, scores = outs[0]
+        gpu_scores = scores.cpu().numpy()
+        idx = [b["first_pair"] + j for j in range(len(b["doc_ids"]))]
+        got, secs, threads = oracle_sample(wl, w_host, doc_m, pairs, idx, args.seed, args.cpu_seconds, dev)
+        cpu = {"value": len(got) / secs, "unit": "pairs/s", "cores": threads, "kind": "oracle",
+               "sample": f"{len(got)} pair(s) of the first timed batch, fp64 C oracle, {secs:.1f} s"}
+        diffs = [abs(float(gpu_scores[p - b["first_pair"]]) - s) for p, s in got.items()]
+        parity = {"pairs": len(diffs), "max_abs_diff": max(diffs), "tolerance": 3e-2,
+                  "oracle_scores": [round(s, 5) for s in got.values()]}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "pairs/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": statistics.mean(step_ms),
+            "p50_batch_ms": statistics.median(step_ms), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic: seeded random-init bf16 weights N(0,0.02), N(0,1) prefix K/V, uniform token ids",
+            "config": {"workload": wl.name,
+                       "model": f"{wl.model.name}: {wl.model.n_layers} layers, hidden {wl.model.hidden}, "
+                                f"{wl.model.n_q_heads}/{wl.model.n_kv_heads} heads, head_dim 128, ffn {wl.model.ffn}",
+                       "docs": wl.n_docs, "m": list(wl.m_choices), "fulldoc_tokens": wl.fulldoc_tokens,
+                       "pairs_per_step": Q * per_q, "queries_per_step": Q, "query_len": [wl.qlen_min, wl.qlen_max],
+                       "candidates": "Zipf(%.1f)" % wl.zipf_s if wl.zipf_s else "uniform",
+                       "parallelism": f"replicas x{world} (pairs sharded by query)",
+                       "l2": "inputs larger than L2 (15 GB of weights streamed per step)"},
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": gpu_launches,
+            "clocks": clk,
+            "latency": {"per_query_pairs": per_q, "p50_ms": lat_sorted[len(lat_sorted) // 2] if lat_sorted else None,
+                        "p90_ms": lat_sorted[int(0.9 * (len(lat_sorted) - 1))] if lat_sorted else None},
+            "kernels": kernels, "parity": parity,
+        }
+        print(json.dumps(line))
+
+
+def run_reference(args, rank, world):
+    """The oracle alone, on the host cores, on bounded samples of the workload."""
+    if rank != 0:
+        return
+    import torch
+
+    from paper_2609_03311_gb300 import synth
+
+    wl = synth.WORKLOADS[args.workload]
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    w = synth.make_weights(wl.model, seed=args.seed, device=dev, norms="ones")
+    w_host = {k: (v.cpu() if isinstance(v, torch.Tensor) else [t.cpu() for t in v]) for k, v in w.items()}
+    del w
+    doc_m = synth.doc_prefix_lengths(wl, seed=args.seed)
+    pairs = build_pairs(wl, args.seed)
+    n_total = args.warmup + args.steps
+    budget = args.cpu_seconds
+    for i in range(args.warmup):
+        oracle_sample(wl, w_host, doc_m, pairs, [i], args.seed, 0.0, dev)
+    done, secs, threads = 0, 0.0, 1
+    for i in range(args.steps):
+        got, s, threads = oracle_sample(wl, w_host, doc_m, pairs, [args.warmup + i], args.seed, budget, dev)
+        done += len(got)
+        secs += s
+    value = done / secs
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "pairs/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic: seeded random-init bf16 weights, N(0,1) prefix K/V, uniform token ids",
+        "config": {"workload": wl.name, "pairs_per_step": 1, "steps_total": n_total},
+        "cpu_baseline": {"value": value, "unit": "pairs/s", "cores": threads, "kind": "oracle",
+                         "sample": f"{done} pair(s), one per step, fp64 C oracle"},
+        "e2e": {"value": value, "unit": "pairs/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def main():
+    args = parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch
+        import torch.distributed as tdist
+
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local_rank)
+        tdist.init_process_group(backend=backend)
+        dist = tdist
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+    else:
+        run_dopr(args, rank, world, local_rank, dist)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

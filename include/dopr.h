@@ -207,6 +207,29 @@ DOPR_API dopr_status dopr_debug_gemm(int32_t M, int32_t N, int32_t K, const void
  */
 DOPR_API dopr_status dopr_debug_wait_timeout(int32_t timeout_ms);
 
+/*
+ * Per-kernel accounting, for measurement.  Every dopr_score call counts its
+ * kernel launches per kernel family (pack, embed_norm, gemm_qkv, qknorm_rope,
+ * attention, gemm_o, rmsnorm, gemm_gate_up, gemm_down, score) together with
+ * the algorithmic floating-point operations and device-memory bytes of those
+ * launches (the minimum the operation needs: each input read once, each output
+ * written once).  While enabled, each launch is also bracketed with CUDA
+ * events on the call's stream and the elapsed device time summed per family.
+ * dopr_profile_enable clears all counters.  dopr_profile_read copies up to
+ * max_entries families into `out` and returns the number of families
+ * (or -1 on a NULL model).
+ */
+typedef struct {
+    char name[24];
+    int64_t launches;
+    double time_ms;   /* summed event time while enabled, else 0 */
+    double flops;     /* algorithmic FLOPs                        */
+    double bytes;     /* algorithmic device-memory bytes           */
+} dopr_kernel_stat;
+
+DOPR_API dopr_status dopr_profile_enable(dopr_model *model, int32_t enable);
+DOPR_API int32_t dopr_profile_read(const dopr_model *model, dopr_kernel_stat *out, int32_t max_entries);
+
 /* Thread-local message describing the last failed call on this thread
  * ("" if none).  The pointer stays valid until the next call on the thread. */
 DOPR_API const char *dopr_last_error(void);

@@ -139,6 +139,8 @@ void free_model(Model* m) {
   dev_free(m->w_o); dev_free(m->mlp_norm); dev_free(m->w_gu); dev_free(m->w_down); dev_free(m->final_norm);
   dev_free(m->score_head); dev_free(m->rope);
   free_workspace(m->ws);
+  for (cudaEvent_t e : m->prof.events) cudaEventDestroy(e);
+  m->prof.events.clear();
 }
 
 void free_store(Store* s) {
@@ -241,6 +243,48 @@ dopr_status map_device_error(int e) {
   return DOPR_OK;
 }
 
+const char* kKindNames[K_COUNT] = {"pack", "embed_norm", "gemm_qkv", "qknorm_rope", "attention",
+                                   "gemm_o", "rmsnorm", "gemm_gate_up", "gemm_down", "score"};
+
+// Launch `fn` as one kernel of family `kind`, counting it and, when profiling
+// is on, bracketing it with CUDA events on `st`.
+template <typename F>
+cudaError_t prof_launch(Model* m, int kind, int n_launches, double flops, double bytes, cudaStream_t st, F&& fn) {
+  Profiler& p = m->prof;
+  p.launches[kind] += n_launches;
+  p.flops[kind] += flops;
+  p.bytes[kind] += bytes;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  if (p.on) {
+    const size_t need = 2 * (p.pending.size() + 1);
+    while (p.events.size() < need) {
+      cudaEvent_t e;
+      cudaError_t r = cudaEventCreate(&e);
+      if (r != cudaSuccess) return r;
+      p.events.push_back(e);
+    }
+    e0 = p.events[need - 2];
+    e1 = p.events[need - 1];
+    cudaEventRecord(e0, st);
+  }
+  cudaError_t r = fn();
+  if (p.on) {
+    cudaEventRecord(e1, st);
+    p.pending.push_back(kind);
+  }
+  return r;
+}
+
+// After the stream has been synchronised: fold the recorded event pairs in.
+void prof_collect(Model* m) {
+  Profiler& p = m->prof;
+  for (size_t i = 0; i < p.pending.size(); ++i) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, p.events[2 * i], p.events[2 * i + 1]) == cudaSuccess) p.ms[p.pending[i]] += ms;
+  }
+  p.pending.clear();
+}
+
 bool same_shape(const dopr_model_config& a, const dopr_model_config& b) {
   return a.n_layers == b.n_layers && a.n_kv_heads == b.n_kv_heads && a.head_dim == b.head_dim;
 }
@@ -308,7 +352,7 @@ dopr_status run_packer(Model* m, Store* s, int32_t n, const int32_t* dqo, const 
   Workspace& w = m->ws;
   CUDA_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), st));
   PackArgs a = pack_args(m, s, n, dqo, dqt, ddoc);
-  CUDA_TRY(launch_pack_order(a, st));
+  CUDA_TRY(prof_launch(m, K_PACK, 4, 0.0, 24.0 * n, st, [&] { return launch_pack_order(a, st); }));
   CUDA_TRY(cudaMemcpyAsync(w.h_tok_off, w.tok_off, sizeof(int32_t) * (n + 1), cudaMemcpyDeviceToHost, st));
   CUDA_TRY(cudaMemcpyAsync(w.h_sorted_slot, w.sorted_slot, sizeof(int32_t) * n, cudaMemcpyDeviceToHost, st));
   CUDA_TRY(cudaMemcpyAsync(w.h_err, w.err, sizeof(int), cudaMemcpyDeviceToHost, st));
@@ -318,7 +362,7 @@ dopr_status run_packer(Model* m, Store* s, int32_t n, const int32_t* dqo, const 
   // token buffers sized from the packed total, then packer part 2
   STATUS_TRY(ensure_call_buffers(m, n, plan.n_tokens, 0, 0));
   a = pack_args(m, s, n, dqo, dqt, ddoc);
-  CUDA_TRY(launch_pack_tokens(a, st));
+  CUDA_TRY(prof_launch(m, K_PACK, 1, 0.0, 16.0 * plan.n_tokens, st, [&] { return launch_pack_tokens(a, st); }));
   // chunks of whole pairs, then attention items (runs of one doc, <= ATTN_MAX_PAIRS)
   const int cap = w.chunk_cap;
   plan.chunk_pair.assign(1, 0);
@@ -354,17 +398,41 @@ dopr_status run_packer(Model* m, Store* s, int32_t n, const int32_t* dqo, const 
 dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cudaStream_t st) {
   Workspace& w = m->ws;
   const auto& c = m->cfg;
-  const int H = c.hidden, F = c.ffn, L = c.n_layers;
+  const int H = c.hidden, F = c.ffn, L = c.n_layers, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
   const int mpad = ((s->max_m + 63) / 64) * 64;
+  const int sms = m->num_sms;
+  auto gemm_cost = [](double M, double N, double K, double out_bytes_per_elem, double n_out) {
+    return std::make_pair(2.0 * M * N * K, (M * K + N * K) * 2.0 + n_out * out_bytes_per_elem);
+  };
   for (size_t ci = 0; ci + 1 < plan.chunk_pair.size(); ++ci) {
     const int32_t s0 = plan.chunk_pair[ci], s1 = plan.chunk_pair[ci + 1];
     const int32_t t0 = w.h_tok_off[s0], Tc = w.h_tok_off[s1] - t0;
-    CUDA_TRY(launch_embed_norm(w.tok_id + t0, Tc, m->embed, m->attn_norm, H, c.rms_eps, w.r, w.xn, st));
+    const double T = Tc;
+    // attention work of this chunk: keys visible per (token, q head) and prefix bytes staged per item
+    double attn_keys = 0.0, prefix_rows = 0.0;
+    for (int32_t sp = s0; sp < s1; ++sp) {
+      const double Tp = w.h_tok_off[sp + 1] - w.h_tok_off[sp];
+      attn_keys += Tp * s->slot_m[w.h_sorted_slot[sp]] + Tp * (Tp + 1) / 2;
+    }
+    for (int32_t it = plan.chunk_item[ci]; it < plan.chunk_item[ci + 1]; ++it) prefix_rows += w.h_items[it].m;
+    const double attn_flops = 4.0 * HEAD_DIM * Hq * attn_keys;
+    const double attn_bytes = T * (2.0 * Hq + 2.0 * Hkv) * HEAD_DIM * 2 + prefix_rows * Hkv * 2 * HEAD_DIM * 2;
+    const auto qkv = gemm_cost(T, m->qkv_dim, H, 2, T * m->qkv_dim);
+    const auto op = gemm_cost(T, H, m->o_dim, 8, T * H);
+    const auto gu = gemm_cost(T, 2.0 * F, H, 2, T * F);
+    const auto dn = gemm_cost(T, H, F, 8, T * H);
+    CUDA_TRY(prof_launch(m, K_EMBED_NORM, 1, 0.0, T * H * 8.0, st, [&] {
+      return launch_embed_norm(w.tok_id + t0, Tc, m->embed, m->attn_norm, H, c.rms_eps, w.r, w.xn, st);
+    }));
     for (int l = 0; l < L; ++l) {
-      CUDA_TRY(launch_gemm(EPI_STORE_BF16, w.tm_xn, m->tm_qkv[l], Tc, m->qkv_dim, H, w.qkv, m->qkv_dim, w.err,
-                           m->num_sms, st));
-      CUDA_TRY(launch_qknorm_rope(w.qkv, Tc, m->qkv_dim, c.n_q_heads, c.n_kv_heads, m->q_norm + (size_t)l * HEAD_DIM,
-                                  m->k_norm + (size_t)l * HEAD_DIM, w.tok_pos + t0, m->rope, c.rms_eps, st));
+      CUDA_TRY(prof_launch(m, K_GEMM_QKV, 1, qkv.first, qkv.second, st, [&] {
+        return launch_gemm(EPI_STORE_BF16, w.tm_xn, m->tm_qkv[l], Tc, m->qkv_dim, H, w.qkv, m->qkv_dim, w.err, sms,
+                           st);
+      }));
+      CUDA_TRY(prof_launch(m, K_QKNORM_ROPE, 1, 0.0, T * (Hq + Hkv) * HEAD_DIM * 4.0, st, [&] {
+        return launch_qknorm_rope(w.qkv, Tc, m->qkv_dim, Hq, Hkv, m->q_norm + (size_t)l * HEAD_DIM,
+                                  m->k_norm + (size_t)l * HEAD_DIM, w.tok_pos + t0, m->rope, c.rms_eps, st);
+      }));
       AttnArgs aa{};
       aa.items = w.items + plan.chunk_item[ci];
       aa.n_items = plan.chunk_item[ci + 1] - plan.chunk_item[ci];
@@ -377,19 +445,33 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       aa.slot_row = s->d_slot_row;
       aa.layer = l;
       aa.n_layers = L;
-      aa.Hq = c.n_q_heads;
-      aa.Hkv = c.n_kv_heads;
+      aa.Hq = Hq;
+      aa.Hkv = Hkv;
       aa.mpad_cap = mpad;
       aa.err = w.err;
-      CUDA_TRY(launch_attention(s->tm_pool, aa, st));
-      CUDA_TRY(launch_gemm(EPI_RESID_ADD_F32, w.tm_o, m->tm_o[l], Tc, H, m->o_dim, w.r, H, w.err, m->num_sms, st));
-      CUDA_TRY(launch_rmsnorm(w.r, Tc, H, m->mlp_norm + (size_t)l * H, c.rms_eps, w.xn, st));
-      CUDA_TRY(launch_gemm(EPI_SWIGLU_BF16, w.tm_xn, m->tm_gu[l], Tc, 2 * F, H, w.act, F, w.err, m->num_sms, st));
-      CUDA_TRY(launch_gemm(EPI_RESID_ADD_F32, w.tm_act, m->tm_down[l], Tc, H, F, w.r, H, w.err, m->num_sms, st));
-      if (l + 1 < L) CUDA_TRY(launch_rmsnorm(w.r, Tc, H, m->attn_norm + (size_t)(l + 1) * H, c.rms_eps, w.xn, st));
+      CUDA_TRY(prof_launch(m, K_ATTENTION, 1, attn_flops, attn_bytes, st,
+                           [&] { return launch_attention(s->tm_pool, aa, st); }));
+      CUDA_TRY(prof_launch(m, K_GEMM_O, 1, op.first, op.second, st, [&] {
+        return launch_gemm(EPI_RESID_ADD_F32, w.tm_o, m->tm_o[l], Tc, H, m->o_dim, w.r, H, w.err, sms, st);
+      }));
+      CUDA_TRY(prof_launch(m, K_RMSNORM, 1, 0.0, T * H * 6.0, st, [&] {
+        return launch_rmsnorm(w.r, Tc, H, m->mlp_norm + (size_t)l * H, c.rms_eps, w.xn, st);
+      }));
+      CUDA_TRY(prof_launch(m, K_GEMM_GATE_UP, 1, gu.first, gu.second, st, [&] {
+        return launch_gemm(EPI_SWIGLU_BF16, w.tm_xn, m->tm_gu[l], Tc, 2 * F, H, w.act, F, w.err, sms, st);
+      }));
+      CUDA_TRY(prof_launch(m, K_GEMM_DOWN, 1, dn.first, dn.second, st, [&] {
+        return launch_gemm(EPI_RESID_ADD_F32, w.tm_act, m->tm_down[l], Tc, H, F, w.r, H, w.err, sms, st);
+      }));
+      if (l + 1 < L)
+        CUDA_TRY(prof_launch(m, K_RMSNORM, 1, 0.0, T * H * 6.0, st, [&] {
+          return launch_rmsnorm(w.r, Tc, H, m->attn_norm + (size_t)(l + 1) * H, c.rms_eps, w.xn, st);
+        }));
     }
-    CUDA_TRY(launch_score(w.r, H, w.tok_off, t0, s0, s1, w.perm, m->final_norm, m->score_head, c.rms_eps, d_scores,
-                          st));
+    CUDA_TRY(prof_launch(m, K_SCORE, 1, 4.0 * H * (s1 - s0), (s1 - s0) * (H * 4.0 + 4.0), st, [&] {
+      return launch_score(w.r, H, w.tok_off, t0, s0, s1, w.perm, m->final_norm, m->score_head, c.rms_eps, d_scores,
+                          st);
+    }));
   }
   return DOPR_OK;
 }
@@ -699,6 +781,7 @@ dopr_status dopr_score(dopr_model* m, dopr_store* s, int32_t n, const int32_t* q
   if (!io_on_device) CUDA_TRY(cudaMemcpyAsync(scores, w.scores, sizeof(float) * n, cudaMemcpyDeviceToHost, st));
   CUDA_TRY(cudaMemcpyAsync(w.h_err, w.err, sizeof(int), cudaMemcpyDeviceToHost, st));
   CUDA_TRY(cudaStreamSynchronize(st));
+  prof_collect(m);
   return map_device_error(*w.h_err);
 }
 
@@ -732,6 +815,7 @@ dopr_status dopr_debug_pack_plan(dopr_model* m, dopr_store* s, int32_t n, const 
   if (tok_id) CUDA_TRY(cudaMemcpy(tok_id, w.tok_id, sizeof(int32_t) * T, cudaMemcpyDeviceToHost));
   if (tok_pair) CUDA_TRY(cudaMemcpy(tok_pair, w.tok_pair, sizeof(int32_t) * T, cudaMemcpyDeviceToHost));
   CUDA_TRY(cudaMemcpy(w.h_err, w.err, sizeof(int), cudaMemcpyDeviceToHost));
+  prof_collect(m);
   return map_device_error(*w.h_err);
 }
 
@@ -762,6 +846,27 @@ dopr_status dopr_debug_gemm(int32_t M, int32_t N, int32_t K, const void* A, cons
   cudaFree(err);
   if (e != cudaSuccess) return fail(DOPR_ERR_CUDA, "gemm failed: %s", cudaGetErrorString(e));
   return map_device_error(h);
+}
+
+dopr_status dopr_profile_enable(dopr_model* m, int32_t enable) {
+  g_last_error.clear();
+  if (!m) return fail(DOPR_ERR_INVALID_ARG, "model is NULL");
+  m->prof.reset();
+  m->prof.on = enable != 0;
+  return DOPR_OK;
+}
+
+int32_t dopr_profile_read(const dopr_model* m, dopr_kernel_stat* out, int32_t max_entries) {
+  if (!m) return -1;
+  for (int k = 0; k < K_COUNT && k < max_entries && out; ++k) {
+    memset(&out[k], 0, sizeof(out[k]));
+    snprintf(out[k].name, sizeof(out[k].name), "%s", kKindNames[k]);
+    out[k].launches = m->prof.launches[k];
+    out[k].time_ms = m->prof.ms[k];
+    out[k].flops = m->prof.flops[k];
+    out[k].bytes = m->prof.bytes[k];
+  }
+  return K_COUNT;
 }
 
 dopr_status dopr_debug_wait_timeout(int32_t timeout_ms) {

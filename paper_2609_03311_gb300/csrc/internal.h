@@ -81,8 +81,26 @@ struct Workspace {
   int64_t h_pair_cap = 0, h_item_cap = 0;
 };
 
+// Per-kernel-family launch counters and (when enabled) CUDA-event timing.
+enum KernelKind : int {
+  K_PACK = 0, K_EMBED_NORM, K_GEMM_QKV, K_QKNORM_ROPE, K_ATTENTION, K_GEMM_O, K_RMSNORM, K_GEMM_GATE_UP,
+  K_GEMM_DOWN, K_SCORE, K_COUNT
+};
+struct Profiler {
+  bool on = false;
+  int64_t launches[K_COUNT] = {};
+  double ms[K_COUNT] = {}, flops[K_COUNT] = {}, bytes[K_COUNT] = {};
+  std::vector<cudaEvent_t> events;  // pairs (start, end), reused across calls
+  std::vector<int> pending;         // kind of each recorded pair
+  void reset() {
+    for (int k = 0; k < K_COUNT; ++k) launches[k] = 0, ms[k] = flops[k] = bytes[k] = 0;
+    pending.clear();
+  }
+};
+
 struct Model {
   dopr_model_config cfg{};
+  Profiler prof;
   int device = 0;
   int num_sms = 0;
   int qkv_dim = 0;  // (Hq + 2 Hkv) * 128

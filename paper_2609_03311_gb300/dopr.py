@@ -33,6 +33,11 @@ class DoprError(RuntimeError):
         super().__init__(f"DOPR_ERR_{name}: {msg}")
 
 
+class KernelStat(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 24), ("launches", ctypes.c_int64), ("time_ms", ctypes.c_double),
+                ("flops", ctypes.c_double), ("bytes", ctypes.c_double)]
+
+
 class ModelConfig(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in ("n_layers", "hidden", "n_q_heads", "n_kv_heads", "head_dim", "ffn",
                                               "vocab", "score_token_id", "max_position")] + \
@@ -65,6 +70,8 @@ def load():
         "dopr_debug_pack_plan": ([P, P, i32, P, P, P, P, P, P, P, P], i32),
         "dopr_debug_gemm": ([i32, i32, i32, P, P, P, i32, P], i32),
         "dopr_debug_wait_timeout": ([i32], i32),
+        "dopr_profile_enable": ([P, i32], i32),
+        "dopr_profile_read": ([P, P, i32], i32),
         "dopr_last_error": ([], ctypes.c_char_p),
         "dopr_version": ([], ctypes.c_char_p),
     }
@@ -238,6 +245,19 @@ def gemm(A: torch.Tensor, B: torch.Tensor, epilogue: int = EPI_STORE_BF16, out: 
     st = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
     _check(load().dopr_debug_gemm(M, N, K, _ptr(A), _ptr(B), _ptr(out), epilogue, st))
     return out
+
+
+def profile_enable(model: Model, on: bool = True):
+    """Clear the per-kernel counters; time each launch with CUDA events while on."""
+    _check(load().dopr_profile_enable(model._h, int(bool(on))))
+
+
+def profile_read(model: Model) -> dict:
+    """{family: {launches, time_ms, flops, bytes}} accumulated since profile_enable."""
+    buf = (KernelStat * 32)()
+    n = load().dopr_profile_read(model._h, buf, 32)
+    return {buf[i].name.decode(): {"launches": int(buf[i].launches), "time_ms": float(buf[i].time_ms),
+                                   "flops": float(buf[i].flops), "bytes": float(buf[i].bytes)} for i in range(n)}
 
 
 def wait_timeout_probe(timeout_ms: int) -> int:
