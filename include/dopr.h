@@ -208,6 +208,35 @@ DOPR_API dopr_status dopr_debug_gemm(int32_t M, int32_t N, int32_t K, const void
 DOPR_API dopr_status dopr_debug_wait_timeout(int32_t timeout_ms);
 
 /*
+ * Allocation-free packing (the paper has no counterpart; this is a service
+ * entry point of this library).  For callers that cannot allocate device
+ * memory while they score -- their GPU memory is owned by another allocator
+ * (e.g. a framework's caching pool), or cudaMalloc/cudaFree would stall a
+ * latency-critical loop by synchronising the device -- this runs the same
+ * device packer ordering step as dopr_score (pairs ordered by (doc_id, input
+ * index), packed token offsets) using only caller buffers and a fixed scratch
+ * array compiled into the library.  It calls no cudaMalloc/cudaFree.
+ *   q_offsets [n_pairs+1] int32, doc_ids [n_pairs] int64: DEVICE memory,
+ *             same meaning as in dopr_score.
+ *   perm      [n_pairs] int32 DEVICE output: input index of sorted pair s.
+ *   tok_off   [n_pairs+1] int32 DEVICE output: first packed token of sorted
+ *             pair s (query tokens + the score token per pair).
+ * Limits: n_pairs <= 32768 and store max_doc_id < 131072; larger requests
+ * return DOPR_ERR_UNSUPPORTED with a message and launch nothing.  The scratch
+ * array (about 768 KiB) is held by every GPU that loads the library until the
+ * process exits.  The first call on a device looks the array's device address
+ * up (cudaGetSymbolAddress) with that device current; make that first call
+ * before any stream capture.  Every call shares the one array: calls that
+ * overlap on the GPU (other streams, other host threads) race and must be
+ * serialised by the caller.  The call runs on cuda_stream (NULL = default)
+ * and returns after its results are written (it synchronises the stream).
+ * Errors: INVALID_ARG, UNKNOWN_DOC, INCOMPLETE, UNSUPPORTED, CUDA.
+ */
+DOPR_API dopr_status dopr_pack_order_noalloc(const dopr_store *store, int32_t n_pairs, const int32_t *q_offsets,
+                                             const int64_t *doc_ids, int32_t *perm, int32_t *tok_off,
+                                             void *cuda_stream);
+
+/*
  * Per-kernel accounting, for measurement.  Every dopr_score call counts its
  * kernel launches per kernel family (pack, embed_norm, gemm_qkv, qknorm_rope,
  * attention, gemm_o, rmsnorm, gemm_gate_up, gemm_down, score) together with

@@ -488,6 +488,8 @@ dopr_status check_ready(Model* m, Store* s) {
 
 }  // namespace
 
+void set_last_error_message(const std::string& msg) { g_last_error = msg; }
+
 bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
                        uint32_t box_cols, uint32_t box_rows, bool swizzle128) {
   auto fn = encode_fn();

@@ -193,6 +193,9 @@ cudaError_t launch_pack_order(const PackArgs& a, cudaStream_t st);
 // Second part, once the token buffers are sized: token ids, positions, pair index.
 cudaError_t launch_pack_tokens(const PackArgs& a, cudaStream_t st);
 
+// Sets the message dopr_last_error() returns on this thread.
+void set_last_error_message(const std::string& msg);
+
 // Debug kernel: bounded wait on a barrier nothing completes.
 cudaError_t launch_wait_timeout_probe(int* err, uint64_t timeout_ns, cudaStream_t st);
 

@@ -70,6 +70,7 @@ def load():
         "dopr_debug_pack_plan": ([P, P, i32, P, P, P, P, P, P, P, P], i32),
         "dopr_debug_gemm": ([i32, i32, i32, P, P, P, i32, P], i32),
         "dopr_debug_wait_timeout": ([i32], i32),
+        "dopr_pack_order_noalloc": ([P, i32, P, P, P, P, P], i32),
         "dopr_profile_enable": ([P, i32], i32),
         "dopr_profile_read": ([P, P, i32], i32),
         "dopr_last_error": ([], ctypes.c_char_p),
@@ -245,6 +246,18 @@ def gemm(A: torch.Tensor, B: torch.Tensor, epilogue: int = EPI_STORE_BF16, out: 
     st = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
     _check(load().dopr_debug_gemm(M, N, K, _ptr(A), _ptr(B), _ptr(out), epilogue, st))
     return out
+
+
+def pack_order_noalloc(store: Store, q_offsets: torch.Tensor, doc_ids: torch.Tensor, perm: torch.Tensor,
+                       tok_off: torch.Tensor, stream=None):
+    """The allocation-free packer ordering step (device tensors in and out)."""
+    assert q_offsets.is_cuda and doc_ids.is_cuda and perm.is_cuda and tok_off.is_cuda
+    assert q_offsets.dtype == torch.int32 and doc_ids.dtype == torch.int64
+    assert perm.dtype == torch.int32 and tok_off.dtype == torch.int32
+    n = q_offsets.numel() - 1
+    st = ctypes.c_void_p(stream.cuda_stream if stream is not None else torch.cuda.current_stream().cuda_stream)
+    _check(load().dopr_pack_order_noalloc(store._h, n, _ptr(q_offsets), _ptr(doc_ids), _ptr(perm), _ptr(tok_off),
+                                          st))
 
 
 def profile_enable(model: Model, on: bool = True):
