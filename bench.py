@@ -375,7 +375,7 @@ def run_dopr(args, rank, world, local_rank, dist):
             "metric": METRIC, "value": value, "unit": "pairs/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": statistics.mean(step_ms),
             "p50_batch_ms": statistics.median(step_ms), "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "bf16",
+            "vs_baseline": None, "dtype": "f16",
             "data": "synthetic: seeded random-init bf16 weights N(0,0.02), N(0,1) prefix K/V, uniform token ids",
             "config": {"workload": wl.name,
                        "model": f"{wl.model.name}: {wl.model.n_layers} layers, hidden {wl.model.hidden}, "

@@ -155,6 +155,10 @@ DOPR_API int64_t dopr_prefix_bytes(const dopr_model_config *cfg, int32_t m);
  *   cuda_stream: a cudaStream_t, or NULL for the default stream.
  *   io_on_device: 0 = the four arrays are host memory (copied in and out by
  *             the call); 1 = device memory (read and written in place).
+ * Arithmetic: the tensor-core operands (activations, projection weights,
+ * q/k/v, attention probabilities) are fp16 -- the bf16 inputs widen to fp16
+ * exactly in its normal range -- with fp32 accumulation, an fp32 residual
+ * stream and fp32 norms, softmax and score head.
  * The call is synchronous in both modes: it synchronises `cuda_stream`
  * once after packing (to size the launches) and once at the end, then
  * reports the device error word.  Pairs of one doc_id are grouped so that
@@ -185,11 +189,11 @@ DOPR_API dopr_status dopr_debug_pack_plan(dopr_model *model, dopr_store *store, 
                                  int32_t *tok_pos, int32_t *tok_id, int32_t *tok_pair);
 
 /*
- * The dense projection kernel alone, for testing: C = A * B^T with A bf16
- * [M][K], B bf16 [N][K] (device pointers), fp32 accumulation.
- *   epilogue 0: out bf16 [M][N] = C
+ * The dense projection kernel alone, for testing: C = A * B^T with A fp16
+ * [M][K], B fp16 [N][K] (IEEE half, device pointers), fp32 accumulation.
+ *   epilogue 0: out fp16 [M][N] = C
  *   epilogue 1: out fp32 [M][N] += C            (residual add)
- *   epilogue 2: out bf16 [M][N/2] = silu(G) * U, where B's rows come in
+ *   epilogue 2: out fp16 [M][N/2] = silu(G) * U, where B's rows come in
  *               blocks of 256: rows 256b..256b+127 are gate rows 128b.., rows
  *               256b+128..256b+255 the matching up rows (SwiGLU, Sec. 4.1 backbone)
  * Requires K % 64 == 0 and N % 256 == 0.  Runs on cuda_stream (NULL = default)

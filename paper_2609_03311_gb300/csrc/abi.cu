@@ -126,6 +126,7 @@ bool kind_is_global(int32_t k) {
 
 void free_workspace(Workspace& w) {
   dev_free(w.r); dev_free(w.xn); dev_free(w.qkv); dev_free(w.o); dev_free(w.act);
+  dev_free(w.ss_e); dev_free(w.ss_a); dev_free(w.ss_m);
   dev_free(w.q_off); dev_free(w.q_tok); dev_free(w.doc_ids); dev_free(w.scores);
   dev_free(w.pair_slot); dev_free(w.perm); dev_free(w.sorted_slot); dev_free(w.tok_off);
   dev_free(w.tok_id); dev_free(w.tok_pos); dev_free(w.tok_pair); dev_free(w.doc_count);
@@ -152,14 +153,14 @@ dopr_status build_weight_maps(Model* m) {
   const int H = c.hidden, F = c.ffn, L = c.n_layers;
   m->tm_qkv.resize(L); m->tm_o.resize(L); m->tm_gu.resize(L); m->tm_down.resize(L);
   for (int l = 0; l < L; ++l) {
-    bool ok = make_tmap_bf16_2d(&m->tm_qkv[l], m->w_qkv + (size_t)l * m->qkv_dim * H, H, m->qkv_dim, (uint64_t)H * 2,
-                                GEMM_BK, GEMM_BN, true) &&
-              make_tmap_bf16_2d(&m->tm_o[l], m->w_o + (size_t)l * H * m->o_dim, m->o_dim, H, (uint64_t)m->o_dim * 2,
-                                GEMM_BK, GEMM_BN, true) &&
-              make_tmap_bf16_2d(&m->tm_gu[l], m->w_gu + (size_t)l * 2 * F * H, H, 2 * F, (uint64_t)H * 2, GEMM_BK,
-                                GEMM_BN, true) &&
-              make_tmap_bf16_2d(&m->tm_down[l], m->w_down + (size_t)l * H * F, F, H, (uint64_t)F * 2, GEMM_BK,
-                                GEMM_BN, true);
+    bool ok = make_tmap_16b_2d(&m->tm_qkv[l], m->w_qkv + (size_t)l * m->qkv_dim * H, H, m->qkv_dim, (uint64_t)H * 2,
+                               GEMM_BK, GEMM_BN, true, true) &&
+              make_tmap_16b_2d(&m->tm_o[l], m->w_o + (size_t)l * H * m->o_dim, m->o_dim, H, (uint64_t)m->o_dim * 2,
+                               GEMM_BK, GEMM_BN, true, true) &&
+              make_tmap_16b_2d(&m->tm_gu[l], m->w_gu + (size_t)l * 2 * F * H, H, 2 * F, (uint64_t)H * 2, GEMM_BK,
+                               GEMM_BN, true, true) &&
+              make_tmap_16b_2d(&m->tm_down[l], m->w_down + (size_t)l * H * F, F, H, (uint64_t)F * 2, GEMM_BK,
+                               GEMM_BN, true, true);
     if (!ok) return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for layer %d weights", l);
   }
   m->maps_ok = true;
@@ -175,11 +176,14 @@ dopr_status alloc_chunk_buffers(Model* m, int cap) {
   STATUS_TRY(dev_alloc(&w.qkv, (size_t)cap * m->qkv_dim));
   STATUS_TRY(dev_alloc(&w.o, (size_t)cap * m->o_dim));
   STATUS_TRY(dev_alloc(&w.act, (size_t)cap * c.ffn));
+  STATUS_TRY(dev_alloc(&w.ss_e, (size_t)cap));
+  STATUS_TRY(dev_alloc(&w.ss_a, (size_t)cap * (c.hidden / GEMM_BN)));
+  STATUS_TRY(dev_alloc(&w.ss_m, (size_t)cap * (c.hidden / GEMM_BN)));
   STATUS_TRY(dev_alloc(&w.err, 1));
   STATUS_TRY(host_alloc(&w.h_err, 1));
-  bool ok = make_tmap_bf16_2d(&w.tm_xn, w.xn, c.hidden, cap, (uint64_t)c.hidden * 2, GEMM_BK, GEMM_BM, true) &&
-            make_tmap_bf16_2d(&w.tm_o, w.o, m->o_dim, cap, (uint64_t)m->o_dim * 2, GEMM_BK, GEMM_BM, true) &&
-            make_tmap_bf16_2d(&w.tm_act, w.act, c.ffn, cap, (uint64_t)c.ffn * 2, GEMM_BK, GEMM_BM, true);
+  bool ok = make_tmap_16b_2d(&w.tm_xn, w.xn, c.hidden, cap, (uint64_t)c.hidden * 2, GEMM_BK, GEMM_BM, true, true) &&
+            make_tmap_16b_2d(&w.tm_o, w.o, m->o_dim, cap, (uint64_t)m->o_dim * 2, GEMM_BK, GEMM_BM, true, true) &&
+            make_tmap_16b_2d(&w.tm_act, w.act, c.ffn, cap, (uint64_t)c.ffn * 2, GEMM_BK, GEMM_BM, true, true);
   if (!ok) return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for activation buffers");
   return DOPR_OK;
 }
@@ -243,7 +247,7 @@ dopr_status map_device_error(int e) {
   return DOPR_OK;
 }
 
-const char* kKindNames[K_COUNT] = {"pack", "embed_norm", "gemm_qkv", "qknorm_rope", "attention",
+const char* kKindNames[K_COUNT] = {"pack", "embed", "gemm_qkv", "qknorm_rope", "attention",
                                    "gemm_o", "rmsnorm", "gemm_gate_up", "gemm_down", "score"};
 
 // Launch `fn` as one kernel of family `kind`, counting it and, when profiling
@@ -399,10 +403,11 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
   Workspace& w = m->ws;
   const auto& c = m->cfg;
   const int H = c.hidden, F = c.ffn, L = c.n_layers, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
+  const int parts = H / GEMM_BN;  // partial sums of squares per row from a residual epilogue
   const int mpad = ((s->max_m + 63) / 64) * 64;
   const int sms = m->num_sms;
-  auto gemm_cost = [](double M, double N, double K, double out_bytes_per_elem, double n_out) {
-    return std::make_pair(2.0 * M * N * K, (M * K + N * K) * 2.0 + n_out * out_bytes_per_elem);
+  auto gemm_cost = [](double M, double N, double K, double out_bytes) {
+    return std::make_pair(2.0 * M * N * K, (M * K + N * K) * 2.0 + out_bytes);
   };
   for (size_t ci = 0; ci + 1 < plan.chunk_pair.size(); ++ci) {
     const int32_t s0 = plan.chunk_pair[ci], s1 = plan.chunk_pair[ci + 1];
@@ -417,22 +422,39 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     for (int32_t it = plan.chunk_item[ci]; it < plan.chunk_item[ci + 1]; ++it) prefix_rows += w.h_items[it].m;
     const double attn_flops = 4.0 * HEAD_DIM * Hq * attn_keys;
     const double attn_bytes = T * (2.0 * Hq + 2.0 * Hkv) * HEAD_DIM * 2 + prefix_rows * Hkv * 2 * HEAD_DIM * 2;
-    const auto qkv = gemm_cost(T, m->qkv_dim, H, 2, T * m->qkv_dim);
-    const auto op = gemm_cost(T, H, m->o_dim, 8, T * H);
-    const auto gu = gemm_cost(T, 2.0 * F, H, 2, T * F);
-    const auto dn = gemm_cost(T, H, F, 8, T * H);
+    // algorithmic bytes: operands once, outputs once (residual: read + write fp32, plus the next norm's bf16 operand)
+    const auto qkv = gemm_cost(T, m->qkv_dim, H, T * m->qkv_dim * 2.0);
+    const auto op = gemm_cost(T, H, m->o_dim, T * H * 10.0);
+    const auto gu = gemm_cost(T, 2.0 * F, H, T * F * 2.0);
+    const auto dn = gemm_cost(T, H, F, T * H * 10.0);
     CUDA_TRY(prof_launch(m, K_EMBED_NORM, 1, 0.0, T * H * 8.0, st, [&] {
-      return launch_embed_norm(w.tok_id + t0, Tc, m->embed, m->attn_norm, H, c.rms_eps, w.r, w.xn, st);
+      return launch_embed(w.tok_id + t0, Tc, m->embed, m->attn_norm, H, c.rms_eps, w.r, w.xn, w.ss_e, st);
     }));
+    GemmParams base{};
+    base.M = Tc;
+    base.norm_dim = H;
+    base.eps = c.rms_eps;
+    base.err = w.err;
     for (int l = 0; l < L; ++l) {
-      CUDA_TRY(prof_launch(m, K_GEMM_QKV, 1, qkv.first, qkv.second, st, [&] {
-        return launch_gemm(EPI_STORE_BF16, w.tm_xn, m->tm_qkv[l], Tc, m->qkv_dim, H, w.qkv, m->qkv_dim, w.err, sms,
-                           st);
-      }));
-      CUDA_TRY(prof_launch(m, K_QKNORM_ROPE, 1, 0.0, T * (Hq + Hkv) * HEAD_DIM * 4.0, st, [&] {
-        return launch_qknorm_rope(w.qkv, Tc, m->qkv_dim, Hq, Hkv, m->q_norm + (size_t)l * HEAD_DIM,
-                                  m->k_norm + (size_t)l * HEAD_DIM, w.tok_pos + t0, m->rope, c.rms_eps, st);
-      }));
+      GemmParams pq = base;  // QKV + attention-norm row scale + q/k norm + RoPE
+      pq.N = m->qkv_dim;
+      pq.K = H;
+      pq.out = w.qkv;
+      pq.ld_out = m->qkv_dim;
+      if (l > 0) {  // layer 0's operand comes from the embedding, already normalised
+        pq.ss_in = w.ss_a;
+        pq.ss_parts = parts;
+        pq.ss_pre = w.ss_m;
+        pq.ss_pre_parts = parts;
+      }
+      pq.tok_pos = w.tok_pos + t0;
+      pq.rope = m->rope;
+      pq.q_norm = m->q_norm + (size_t)l * HEAD_DIM;
+      pq.k_norm = m->k_norm + (size_t)l * HEAD_DIM;
+      pq.q_cols = Hq * HEAD_DIM;
+      pq.k_cols = Hkv * HEAD_DIM;
+      CUDA_TRY(prof_launch(m, K_GEMM_QKV, 1, qkv.first, qkv.second, st,
+                           [&] { return launch_gemm(EPI_QKV, w.tm_xn, m->tm_qkv[l], pq, sms, st); }));
       AttnArgs aa{};
       aa.items = w.items + plan.chunk_item[ci];
       aa.n_items = plan.chunk_item[ci + 1] - plan.chunk_item[ci];
@@ -451,22 +473,45 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       aa.err = w.err;
       CUDA_TRY(prof_launch(m, K_ATTENTION, 1, attn_flops, attn_bytes, st,
                            [&] { return launch_attention(s->tm_pool, aa, st); }));
-      CUDA_TRY(prof_launch(m, K_GEMM_O, 1, op.first, op.second, st, [&] {
-        return launch_gemm(EPI_RESID_ADD_F32, w.tm_o, m->tm_o[l], Tc, H, m->o_dim, w.r, H, w.err, sms, st);
-      }));
-      CUDA_TRY(prof_launch(m, K_RMSNORM, 1, 0.0, T * H * 6.0, st, [&] {
-        return launch_rmsnorm(w.r, Tc, H, m->mlp_norm + (size_t)l * H, c.rms_eps, w.xn, st);
-      }));
-      CUDA_TRY(prof_launch(m, K_GEMM_GATE_UP, 1, gu.first, gu.second, st, [&] {
-        return launch_gemm(EPI_SWIGLU_BF16, w.tm_xn, m->tm_gu[l], Tc, 2 * F, H, w.act, F, w.err, sms, st);
-      }));
-      CUDA_TRY(prof_launch(m, K_GEMM_DOWN, 1, dn.first, dn.second, st, [&] {
-        return launch_gemm(EPI_RESID_ADD_F32, w.tm_act, m->tm_down[l], Tc, H, F, w.r, H, w.err, sms, st);
-      }));
-      if (l + 1 < L)
-        CUDA_TRY(prof_launch(m, K_RMSNORM, 1, 0.0, T * H * 6.0, st, [&] {
-          return launch_rmsnorm(w.r, Tc, H, m->attn_norm + (size_t)(l + 1) * H, c.rms_eps, w.xn, st);
-        }));
+      GemmParams po = base;  // O projection + residual, emits the MLP norm's operand
+      po.N = H;
+      po.K = m->o_dim;
+      po.out = w.r;
+      po.ld_out = H;
+      po.xn_out = w.xn;
+      po.xn_gain = m->mlp_norm + (size_t)l * H;
+      po.ss_out = w.ss_m;
+      po.ss_out_parts = parts;
+      po.ss_pre = l == 0 ? w.ss_e : w.ss_a;  // the attention norm of this layer
+      po.ss_pre_parts = l == 0 ? 1 : parts;
+      CUDA_TRY(prof_launch(m, K_GEMM_O, 1, op.first, op.second, st,
+                           [&] { return launch_gemm(EPI_RESID_ADD, w.tm_o, m->tm_o[l], po, sms, st); }));
+      GemmParams pg = base;  // gate/up + MLP-norm row scale + SwiGLU
+      pg.N = 2 * F;
+      pg.K = H;
+      pg.out = w.act;
+      pg.ld_out = F;
+      pg.ss_in = w.ss_m;
+      pg.ss_parts = parts;
+      pg.ss_pre = po.ss_pre;
+      pg.ss_pre_parts = po.ss_pre_parts;
+      CUDA_TRY(prof_launch(m, K_GEMM_GATE_UP, 1, gu.first, gu.second, st,
+                           [&] { return launch_gemm(EPI_SWIGLU, w.tm_xn, m->tm_gu[l], pg, sms, st); }));
+      GemmParams pd = base;  // down projection + residual, emits the next attention norm's operand
+      pd.N = H;
+      pd.K = F;
+      pd.out = w.r;
+      pd.ld_out = H;
+      if (l + 1 < L) {
+        pd.xn_out = w.xn;
+        pd.xn_gain = m->attn_norm + (size_t)(l + 1) * H;
+        pd.ss_out = w.ss_a;
+        pd.ss_out_parts = parts;
+        pd.ss_pre = w.ss_m;  // the MLP norm of this layer
+        pd.ss_pre_parts = parts;
+      }
+      CUDA_TRY(prof_launch(m, K_GEMM_DOWN, 1, dn.first, dn.second, st,
+                           [&] { return launch_gemm(EPI_RESID_ADD, w.tm_act, m->tm_down[l], pd, sms, st); }));
     }
     CUDA_TRY(prof_launch(m, K_SCORE, 1, 4.0 * H * (s1 - s0), (s1 - s0) * (H * 4.0 + 4.0), st, [&] {
       return launch_score(w.r, H, w.tok_off, t0, s0, s1, w.perm, m->final_norm, m->score_head, c.rms_eps, d_scores,
@@ -490,15 +535,16 @@ dopr_status check_ready(Model* m, Store* s) {
 
 void set_last_error_message(const std::string& msg) { g_last_error = msg; }
 
-bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
-                       uint32_t box_cols, uint32_t box_rows, bool swizzle128) {
+bool make_tmap_16b_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
+                      uint32_t box_cols, uint32_t box_rows, bool swizzle128, bool half) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {row_stride_bytes};
   cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+  CUresult r = fn(map, half ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                  const_cast<void*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE,
                   swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -591,20 +637,25 @@ dopr_status dopr_model_put_weight(dopr_model* m, int32_t kind, int32_t layer, co
   const size_t l = (size_t)layer;
   const cudaMemcpyKind dir = src_on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
   int64_t expect = 0;
-  bf16* dst = nullptr;
+  void* dst = nullptr;
+  bool matrix = false;  // projection matrices are held as fp16 for the tensor cores
   switch (kind) {
     case DOPR_W_EMBED: expect = (int64_t)c.vocab * H; dst = m->embed; break;
     case DOPR_W_ATTN_NORM: expect = H; dst = m->attn_norm + l * H; break;
-    case DOPR_W_Q: expect = Hq * D * H; dst = m->w_qkv + l * m->qkv_dim * H; break;
-    case DOPR_W_K: expect = Hkv * D * H; dst = m->w_qkv + (l * m->qkv_dim + Hq * D) * H; break;
-    case DOPR_W_V: expect = Hkv * D * H; dst = m->w_qkv + (l * m->qkv_dim + (Hq + Hkv) * D) * H; break;
+    case DOPR_W_Q: expect = Hq * D * H; dst = m->w_qkv + l * m->qkv_dim * H; matrix = true; break;
+    case DOPR_W_K: expect = Hkv * D * H; dst = m->w_qkv + (l * m->qkv_dim + Hq * D) * H; matrix = true; break;
+    case DOPR_W_V: expect = Hkv * D * H; dst = m->w_qkv + (l * m->qkv_dim + (Hq + Hkv) * D) * H; matrix = true; break;
     case DOPR_W_Q_NORM: expect = D; dst = m->q_norm + l * D; break;
     case DOPR_W_K_NORM: expect = D; dst = m->k_norm + l * D; break;
-    case DOPR_W_O: expect = H * Hq * D; dst = m->w_o + l * H * m->o_dim; break;
+    case DOPR_W_O: expect = H * Hq * D; dst = m->w_o + l * H * m->o_dim; matrix = true; break;
     case DOPR_W_MLP_NORM: expect = H; dst = m->mlp_norm + l * H; break;
     case DOPR_W_GATE:
-    case DOPR_W_UP: expect = F * H; dst = m->w_gu + l * 2 * F * H + (kind == DOPR_W_UP ? 128 * H : 0); break;
-    case DOPR_W_DOWN: expect = H * F; dst = m->w_down + l * H * F; break;
+    case DOPR_W_UP:
+      expect = F * H;
+      dst = m->w_gu + l * 2 * F * H + (kind == DOPR_W_UP ? 128 * H : 0);
+      matrix = true;
+      break;
+    case DOPR_W_DOWN: expect = H * F; dst = m->w_down + l * H * F; matrix = true; break;
     case DOPR_W_FINAL_NORM: expect = H; dst = m->final_norm; break;
     case DOPR_W_SCORE_HEAD: expect = 2 * H; dst = m->score_head; break;
   }
@@ -612,11 +663,22 @@ dopr_status dopr_model_put_weight(dopr_model* m, int32_t kind, int32_t layer, co
     return fail(DOPR_ERR_INVALID_ARG, "weight kind %d: %lld elements given, %lld expected", kind, (long long)n_elems,
                 (long long)expect);
   CUDA_TRY(cudaSetDevice(m->device));
-  if (kind == DOPR_W_GATE || kind == DOPR_W_UP) {
-    // rows 128b..128b+127 of the source go to rows 256b (+128 for up) of the fused matrix
-    CUDA_TRY(cudaMemcpy2D(dst, 256 * H * 2, src, 128 * H * 2, 128 * H * 2, F / 128, dir));
-  } else {
+  if (!matrix) {
     CUDA_TRY(cudaMemcpy(dst, src, (size_t)expect * 2, dir));
+  } else {
+    // stage, widen bf16 -> fp16 (exact in fp16's normal range), then place
+    void* stage = nullptr;
+    CUDA_TRY(cudaMalloc(&stage, (size_t)expect * 2));
+    cudaError_t e = cudaMemcpy(stage, src, (size_t)expect * 2, dir);
+    if (e == cudaSuccess) e = launch_bf16_to_f16(stage, expect, 0);
+    if (e == cudaSuccess) {
+      if (kind == DOPR_W_GATE || kind == DOPR_W_UP)  // rows 128b.. go to rows 256b (+128 for up)
+        e = cudaMemcpy2D(dst, 256 * H * 2, stage, 128 * H * 2, 128 * H * 2, F / 128, cudaMemcpyDeviceToDevice);
+      else
+        e = cudaMemcpy(dst, stage, (size_t)expect * 2, cudaMemcpyDeviceToDevice);
+    }
+    cudaFree(stage);
+    if (e != cudaSuccess) return fail(DOPR_ERR_CUDA, "weight upload failed: %s", cudaGetErrorString(e));
   }
   m->have[(size_t)kind * c.n_layers + l] = 1;
   return DOPR_OK;
@@ -660,7 +722,8 @@ dopr_status dopr_store_create(const dopr_model_config* cfg, int64_t max_doc_id, 
       guard(fail(DOPR_ERR_CUDA, "store initialisation failed"));
   }
   if (st == DOPR_OK &&
-      !make_tmap_bf16_2d(&s->tm_pool, s->pool, HEAD_DIM, std::max<int64_t>(s->pool_rows, 1), HEAD_DIM * 2, 64, 64, true))
+      !make_tmap_16b_2d(&s->tm_pool, s->pool, HEAD_DIM, std::max<int64_t>(s->pool_rows, 1), HEAD_DIM * 2, 64, 64, true,
+                        false))
     guard(fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for the store pool"));
   if (st != DOPR_OK) {
     free_store(s);
@@ -830,8 +893,8 @@ dopr_status dopr_debug_gemm(int32_t M, int32_t N, int32_t K, const void* A, cons
   if (M == 0) return DOPR_OK;
   if (gemm_setup() != cudaSuccess) return fail(DOPR_ERR_CUDA, "gemm setup failed");
   CUtensorMap ta, tb;
-  if (!make_tmap_bf16_2d(&ta, A, K, M, (uint64_t)K * 2, GEMM_BK, GEMM_BM, true) ||
-      !make_tmap_bf16_2d(&tb, B, K, N, (uint64_t)K * 2, GEMM_BK, GEMM_BN, true))
+  if (!make_tmap_16b_2d(&ta, A, K, M, (uint64_t)K * 2, GEMM_BK, GEMM_BM, true, true) ||
+      !make_tmap_16b_2d(&tb, B, K, N, (uint64_t)K * 2, GEMM_BK, GEMM_BN, true, true))
     return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed (pointers must be 16-byte aligned)");
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
@@ -840,8 +903,14 @@ dopr_status dopr_debug_gemm(int32_t M, int32_t N, int32_t K, const void* A, cons
   int* err = nullptr;
   CUDA_TRY(cudaMalloc(&err, sizeof(int)));
   cudaMemsetAsync(err, 0, sizeof(int), st);
-  const int64_t ld = epilogue == EPI_SWIGLU_BF16 ? N / 2 : N;
-  cudaError_t e = launch_gemm(epilogue, ta, tb, M, N, K, out, ld, err, sms, st);
+  GemmParams gp{};
+  gp.M = M;
+  gp.N = N;
+  gp.K = K;
+  gp.out = out;
+  gp.ld_out = epilogue == EPI_SWIGLU ? N / 2 : N;
+  gp.err = err;
+  cudaError_t e = launch_gemm(epilogue, ta, tb, gp, sms, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   int h = 0;
   if (e == cudaSuccess) e = cudaMemcpy(&h, err, sizeof(int), cudaMemcpyDeviceToHost);

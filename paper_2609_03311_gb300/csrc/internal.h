@@ -15,6 +15,7 @@
 namespace dopr {
 
 typedef __nv_bfloat16 bf16;
+typedef __half f16;  // tensor-core operand type of the scoring pass (fp32 accumulation)
 
 constexpr int HEAD_DIM = 128;
 constexpr int MAX_PREFIX = 256;       // largest m the store accepts
@@ -52,10 +53,13 @@ struct Store {
 struct Workspace {
   int chunk_cap = 0;  // tokens per chunk
   float* r = nullptr;          // [chunk][H] fp32 residual stream
-  bf16* xn = nullptr;          // [chunk][H] normed activations
-  bf16* qkv = nullptr;         // [chunk][(Hq+2Hkv)*128]
-  bf16* o = nullptr;           // [chunk][Hq*128]
-  bf16* act = nullptr;         // [chunk][F]
+  f16* xn = nullptr;           // [chunk][H] norm operand (see GemmParams)
+  f16* qkv = nullptr;          // [chunk][(Hq+2Hkv)*128] q, k after norm+RoPE, v
+  f16* o = nullptr;            // [chunk][Hq*128] attention output
+  f16* act = nullptr;          // [chunk][F] SwiGLU output
+  float* ss_e = nullptr;       // [chunk] sum of squares of the embedded rows
+  float* ss_a = nullptr;       // [chunk][H/256] partial sums of squares for the attention norm
+  float* ss_m = nullptr;       // [chunk][H/256] partial sums of squares for the MLP norm
   CUtensorMap tm_xn{}, tm_o{}, tm_act{};
   // per call, grown on demand
   int64_t pair_cap = 0, tok_cap = 0, qtok_cap = 0, doc_cap = 0, item_cap = 0;
@@ -107,13 +111,13 @@ struct Model {
   int o_dim = 0;    // Hq * 128
   bf16* embed = nullptr;       // [V][H]
   bf16* attn_norm = nullptr;   // [L][H]
-  bf16* w_qkv = nullptr;       // [L][qkv_dim][H]
+  f16* w_qkv = nullptr;        // [L][qkv_dim][H]   (projection matrices held as fp16)
   bf16* q_norm = nullptr;      // [L][128]
   bf16* k_norm = nullptr;      // [L][128]
-  bf16* w_o = nullptr;         // [L][H][o_dim]
+  f16* w_o = nullptr;          // [L][H][o_dim]
   bf16* mlp_norm = nullptr;    // [L][H]
-  bf16* w_gu = nullptr;        // [L][2F][H], gate/up interleaved in 128-row blocks
-  bf16* w_down = nullptr;      // [L][H][F]
+  f16* w_gu = nullptr;         // [L][2F][H], gate/up interleaved in 128-row blocks
+  f16* w_down = nullptr;       // [L][H][F]
   bf16* final_norm = nullptr;  // [H]
   bf16* score_head = nullptr;  // [2][H]
   float2* rope = nullptr;      // [max_position][64] (cos, sin)
@@ -125,23 +129,52 @@ struct Model {
 
 // ------------------------------------------------------------ launchers
 // Tensor map helper (driver entry point resolved at run time).
-bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
-                       uint32_t box_cols, uint32_t box_rows, bool swizzle128);
+// 2-D map over 16-bit elements (fp16 when `half` is set, else bf16).
+bool make_tmap_16b_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
+                      uint32_t box_cols, uint32_t box_rows, bool swizzle128, bool half);
 
 // GEMM epilogues.
-enum GemmEpi : int { EPI_STORE_BF16 = 0, EPI_RESID_ADD_F32 = 1, EPI_SWIGLU_BF16 = 2 };
+enum GemmEpi : int { EPI_STORE = 0, EPI_RESID_ADD = 1, EPI_SWIGLU = 2, EPI_QKV = 3 };
 constexpr int GEMM_BM = 128, GEMM_BN = 256, GEMM_BK = 64;
+struct GemmParams {
+  int M, N, K;
+  void* out;          // fp16 [M][ld_out] (store, QKV, SwiGLU: ld_out = N/2) or fp32 residual [M][ld_out]
+  int64_t ld_out;
+  // Fused RMSNorm.  rs(ss, parts) = rsqrt(sum_i ss[row*parts + i] / norm_dim + eps); a null
+  // array means 1.  Producer (residual epilogue): xn_out = f16(r' * xn_gain * rs(ss_pre)) and
+  // ss_out[row*ss_out_parts + n-tile] = partial sum of r'^2.  Consumer: accumulator rows are
+  // scaled by rs(ss_in) / rs(ss_pre), so the operand stays near unit scale in fp16.
+  const float* ss_in;
+  int ss_parts;
+  const float* ss_pre;
+  int ss_pre_parts;
+  int norm_dim;
+  float eps;
+  f16* xn_out;
+  const bf16* xn_gain;
+  float* ss_out;
+  int ss_out_parts;
+  // QKV epilogue: per-head RMSNorm gains and RoPE at tok_pos[row]
+  const int32_t* tok_pos;
+  const float2* rope;
+  const bf16* q_norm;
+  const bf16* k_norm;
+  int q_cols, k_cols;
+  int* err;
+  uint64_t timeout_ns;
+};
 cudaError_t gemm_setup();
-// C[M][N] = A[M][K] * B[N][K]^T with the given epilogue writing `out` (ld in elements).
-cudaError_t launch_gemm(int epi, const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
-                        int64_t ld_out, int* err, int num_sms, cudaStream_t st);
+// C[M][N] = A[M][K] * B[N][K]^T followed by the epilogue `epi`.
+cudaError_t launch_gemm(int epi, const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p, int num_sms,
+                        cudaStream_t st);
 
 // Row kernels.
-cudaError_t launch_embed_norm(const int32_t* tok_id, int T, const bf16* embed, const bf16* gain, int H, float eps,
-                              float* r, bf16* xn, cudaStream_t st);
-cudaError_t launch_rmsnorm(const float* r, int T, int H, const bf16* gain, float eps, bf16* xn, cudaStream_t st);
-cudaError_t launch_qknorm_rope(bf16* qkv, int T, int ld, int Hq, int Hkv, const bf16* qn, const bf16* kn,
-                               const int32_t* tok_pos, const float2* rope, float eps, cudaStream_t st);
+// r[t] = E[tok_id[t]] (fp32), ss[t] = sum(r[t]^2), xn[t] = f16(r[t] * rsqrt(ss[t]/H + eps) * gain):
+// the embedding and the first RMSNorm.
+cudaError_t launch_embed(const int32_t* tok_id, int T, const bf16* embed, const bf16* gain, int H, float eps, float* r,
+                         f16* xn, float* ss, cudaStream_t st);
+// In place: n bf16 values -> fp16 (saturating at +-65504).
+cudaError_t launch_bf16_to_f16(void* buf, int64_t n, cudaStream_t st);
 cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end,
                          const int32_t* perm, const bf16* gain, const bf16* head, float eps, float* scores,
                          cudaStream_t st);
@@ -154,9 +187,9 @@ struct AttnArgs {
   int n_items;
   const int32_t* tok_off;  // sorted pair -> first packed token
   int32_t tok0;            // first packed token of this chunk
-  const bf16* qkv;
+  const f16* qkv;
   int ld_qkv;
-  bf16* out;
+  f16* out;
   int ld_out;
   const int64_t* slot_row;
   int layer, n_layers, Hq, Hkv;

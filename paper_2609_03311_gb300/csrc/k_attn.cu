@@ -10,7 +10,8 @@
 // one kv head interleaved, so a 16-row warp tile covers 16/G tokens x G heads.
 // Per 64-row block the warps sweep the prefix blocks, then stream the pair's
 // own keys 0..j in 64-key chunks (cp.async, zero-filled past the end).
-// Scores and P.V use warp-level bf16 mma with fp32 accumulation; the softmax
+// Scores and P.V use warp-level fp16 mma with fp32 accumulation (the stored
+// bf16 prefix is widened to fp16 in shared memory after it lands); the softmax
 // is the online (running max / running sum) form with quad shuffles.
 #include <math.h>
 
@@ -57,8 +58,8 @@ __device__ __forceinline__ void attend_block(uint32_t kbase, uint32_t vbase, int
       const int c = 2 * ks + ((lane >> 3) & 1);
       uint32_t b0, b1, b2, b3;
       ldmatrix_x4(kbase + off64(key, c), b0, b1, b2, b3);
-      mma_bf16_16816(s[2 * np], qf[ks], b0, b1);
-      mma_bf16_16816(s[2 * np + 1], qf[ks], b2, b3);
+      mma_f16_16816(s[2 * np], qf[ks], b0, b1);
+      mma_f16_16816(s[2 * np + 1], qf[ks], b2, b3);
     }
   }
   float mx[2] = {-INFINITY, -INFINITY};
@@ -104,18 +105,18 @@ __device__ __forceinline__ void attend_block(uint32_t kbase, uint32_t vbase, int
 #pragma unroll
   for (int kk = 0; kk < 4; ++kk) {
     uint32_t a[4];
-    a[0] = pack_bf16x2(s[2 * kk][0], s[2 * kk][1]);
-    a[1] = pack_bf16x2(s[2 * kk][2], s[2 * kk][3]);
-    a[2] = pack_bf16x2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-    a[3] = pack_bf16x2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
+    a[0] = pack_f16x2(s[2 * kk][0], s[2 * kk][1]);
+    a[1] = pack_f16x2(s[2 * kk][2], s[2 * kk][3]);
+    a[2] = pack_f16x2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
+    a[3] = pack_f16x2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
 #pragma unroll
     for (int dp = 0; dp < 8; ++dp) {
       const int key = kk * 16 + (lane & 7) + (((lane >> 3) & 1) << 3);
       const int c = 2 * dp + (lane >> 4);
       uint32_t b0, b1, b2, b3;
       ldmatrix_x4_trans(vbase + off64(key, c), b0, b1, b2, b3);
-      mma_bf16_16816(o[2 * dp], a, b0, b1);
-      mma_bf16_16816(o[2 * dp + 1], a, b2, b3);
+      mma_f16_16816(o[2 * dp], a, b0, b1);
+      mma_f16_16816(o[2 * dp + 1], a, b2, b3);
     }
   }
 }
@@ -161,20 +162,30 @@ __global__ void __launch_bounds__(THREADS) k_attn(const __grid_constant__ CUtens
       if (tid == 0) mbar_wait(bar, 0, a.err, 100000000ull);  // let the copies land first
       return;
     }
-    // rows m .. nbox*64-1 of the boxes hold other data: zero them so masked
-    // keys contribute exactly 0 to P.V
-    const int pad = nbox * 64 - m;
+    // The stored prefix is bf16: widen it to fp16 in place (element-wise, so the
+    // swizzled layout is unchanged).  Rows m .. nbox*64-1 of the boxes hold other
+    // data: zero them so masked keys contribute exactly 0 to P.V.
     uint8_t* gk = smem;
     uint8_t* gv = smem + a.mpad_cap * ROW_BYTES;
-    for (int i = tid; i < pad * 16; i += THREADS) {
-      const int r = m + i / 16, c = i % 16;
-      *reinterpret_cast<uint4*>(gk + off64(r, c)) = make_uint4(0, 0, 0, 0);
-      *reinterpret_cast<uint4*>(gv + off64(r, c)) = make_uint4(0, 0, 0, 0);
+    for (int i = tid; i < nbox * 64 * 16; i += THREADS) {
+      const int r = i / 16, c = i % 16;
+      uint4* pk = reinterpret_cast<uint4*>(gk + off64(r, c));
+      uint4* pv = reinterpret_cast<uint4*>(gv + off64(r, c));
+      if (r >= m) {
+        *pk = make_uint4(0, 0, 0, 0);
+        *pv = make_uint4(0, 0, 0, 0);
+      } else {
+        uint4 x = *pk, y = *pv;
+        x = make_uint4(bf16x2_to_f16x2(x.x), bf16x2_to_f16x2(x.y), bf16x2_to_f16x2(x.z), bf16x2_to_f16x2(x.w));
+        y = make_uint4(bf16x2_to_f16x2(y.x), bf16x2_to_f16x2(y.y), bf16x2_to_f16x2(y.z), bf16x2_to_f16x2(y.w));
+        *pk = x;
+        *pv = y;
+      }
     }
     __syncthreads();
   }
 
-  const bf16* qkv = a.qkv;
+  const f16* qkv = a.qkv;
   const int ld = a.ld_qkv;
   const int kcol = (a.Hq + g) * HEAD_DIM;
   const int vcol = (a.Hq + a.Hkv + g) * HEAD_DIM;
@@ -196,7 +207,7 @@ __global__ void __launch_bounds__(THREADS) k_attn(const __grid_constant__ CUtens
           const int row = row0 + r;
           const bool ok = row < R;
           const int j = ok ? row / G : 0, hh = ok ? row % G : 0;
-          const bf16* src = qkv + static_cast<int64_t>(tb + j) * ld + (g * G + hh) * HEAD_DIM + c * 8;
+          const f16* src = qkv + static_cast<int64_t>(tb + j) * ld + (g * G + hh) * HEAD_DIM + c * 8;
           cp_async16(sQ + off16(r, c), src, ok);
         }
       }
@@ -235,7 +246,7 @@ __global__ void __launch_bounds__(THREADS) k_attn(const __grid_constant__ CUtens
           const int kv = idx >> 10, rem = idx & 1023, key = rem >> 4, c = rem & 15;
           const bool ok = c0 + key <= jmax;
           const int row = tb + (ok ? c0 + key : 0);
-          const bf16* src = qkv + static_cast<int64_t>(row) * ld + (kv ? vcol : kcol) + c * 8;
+          const f16* src = qkv + static_cast<int64_t>(row) * ld + (kv ? vcol : kcol) + c * 8;
           cp_async16((kv ? sOV : sOK) + off64(key, c), src, ok);
         }
         cp_async_commit();
@@ -257,11 +268,11 @@ __global__ void __launch_bounds__(THREADS) k_attn(const __grid_constant__ CUtens
           const int row = row0 + (lane >> 2) + hr * 8;
           if (row < R) {
             const int j = row / G, hh = row % G;
-            bf16* dst = a.out + static_cast<int64_t>(tb + j) * a.ld_out + (g * G + hh) * HEAD_DIM + (lane & 3) * 2;
+            f16* dst = a.out + static_cast<int64_t>(tb + j) * a.ld_out + (g * G + hh) * HEAD_DIM + (lane & 3) * 2;
             const float inv = hr ? inv1 : inv0;
 #pragma unroll
             for (int dt = 0; dt < 16; ++dt)
-              *reinterpret_cast<uint32_t*>(dst + dt * 8) = pack_bf16x2(o[dt][2 * hr] * inv, o[dt][2 * hr + 1] * inv);
+              *reinterpret_cast<uint32_t*>(dst + dt * 8) = pack_f16x2(o[dt][2 * hr] * inv, o[dt][2 * hr + 1] * inv);
           }
         }
       }

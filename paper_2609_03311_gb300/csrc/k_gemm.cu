@@ -1,6 +1,6 @@
 // k_gemm.cu -- dense projections of the decoder (QKV, O, gate/up, down) on
-// the 5th-generation tensor cores: C[M][N] = A[M][K] * B[N][K]^T, bf16 in,
-// fp32 accumulate in tensor memory, fused epilogues.
+// the 5th-generation tensor cores: C[M][N] = A[M][K] * B[N][K]^T, fp16
+// operands, fp32 accumulate in tensor memory, fused epilogues.
 //
 // Design (sm_103a, one CTA per SM, persistent):
 //   warp 0      TMA producer: 128x64 A tile + 256x64 B tile per stage, 128-byte
@@ -8,11 +8,25 @@
 //   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and one
 //               elected thread issues tcgen05.mma (M=128, N=256, K=16) per k-step,
 //               committing stage releases and accumulator-ready barriers;
-//   warps 2..5  epilogue: tcgen05.ld rows of the finished accumulator (one TMEM lane
-//               quarter per warp, one output row per thread), apply the epilogue and
-//               store, then release the accumulator so the next tile's MMAs overlap.
+//   warps 2..5  epilogue: tcgen05.ld the finished accumulator (one TMEM lane quarter
+//               = 32 rows per warp, one row per thread), apply the epilogue in that
+//               row-per-thread layout, then transpose 32x32-word chunks through
+//               padded shared memory so every global access is a 128-byte row
+//               segment written by 8 consecutive lanes; finally release the
+//               accumulator so the next tile's MMAs overlap the epilogue.
 // Tiles are visited in groups of 16 M-blocks so the weight tiles a wave reads
 // stay in L2 while the activation rows of the group are reused across N.
+//
+// Fused epilogues (the decoder's RMSNorms live here, not in separate kernels):
+//   RMSNorm(r) * g = rs * (r (.) g) with rs = rsqrt(mean(r^2) + eps).  The
+//   residual-add epilogue writes r' = r + C, the next GEMM's operand
+//   f16(r' (.) g_next * rs_pre) -- rs_pre is the row's previous norm factor,
+//   which keeps the operand near unit scale -- and, per row and 256-column
+//   tile, the partial sum of r'^2.  The consuming GEMM sums those partials
+//   (in a fixed order) and scales its accumulator rows by rs / rs_pre.
+//   QKV epilogue: row scale, then per 128-column q/k head RMSNorm with the
+//   q/k gain and rotate-half RoPE at the token's position (pairs i, i+64).
+//   SwiGLU epilogue: silu(rs * gate) * (rs * up).
 // Every barrier wait is bounded (DEV_ERR_TIMEOUT) and the kernel always drains
 // its own copies and MMAs and frees TMEM before returning.
 #include "device_common.cuh"
@@ -28,18 +42,13 @@ constexpr int B_BYTES = BN * BK * 2;  // 32 KiB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 2 * BN;     // two accumulators
 constexpr int THREADS = 192;
+constexpr int EPI_WARPS = 4;
 constexpr int GROUP_M = 16;
+constexpr int XPOSE_WORDS = 32 * 33;  // per epilogue warp: 32 rows x 32 words, padded row stride 33
+constexpr int XPOSE_BYTES = EPI_WARPS * XPOSE_WORDS * 4;
 constexpr int BAR_BYTES = 256;
-constexpr int SMEM_BYTES = 1024 /*alignment slack*/ + STAGES * STAGE_BYTES + BAR_BYTES;
-constexpr uint32_t IDESC = umma_idesc_bf16(BM, BN);
-
-struct GemmParams {
-  int M, N, K;
-  void* out;
-  int64_t ld_out;
-  int* err;
-  uint64_t timeout_ns;
-};
+constexpr int SMEM_BYTES = 1024 /*alignment slack*/ + STAGES * STAGE_BYTES + XPOSE_BYTES + BAR_BYTES;
+constexpr uint32_t IDESC = umma_idesc_f16(BM, BN);
 
 __device__ __forceinline__ void tile_coords(int t, int m_tiles, int n_tiles, int& mb, int& nb) {
   const int group = GROUP_M * n_tiles;
@@ -53,74 +62,212 @@ __device__ __forceinline__ void tile_coords(int t, int m_tiles, int n_tiles, int
 
 __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + __expf(-x)); }
 
+// RMSNorm factor of a row from its partial sums of squares (fixed summation order).
+__device__ __forceinline__ float norm_factor(const float* ss, int parts, const GemmParams& p, int row) {
+  if (!ss) return 1.f;
+  const float* s = ss + static_cast<int64_t>(min(row, p.M - 1)) * parts;
+  float t = 0.f;
+  for (int i = 0; i < parts; ++i) t += s[i];
+  return rsqrtf(t / static_cast<float>(p.norm_dim) + p.eps);
+}
+// Consumer-side row scale: the operand was written as r * g * rs(ss_pre).
+__device__ __forceinline__ float row_scale(const GemmParams& p, int row) {
+  return norm_factor(p.ss_in, p.ss_parts, p, row) / norm_factor(p.ss_pre, p.ss_pre_parts, p, row);
+}
+
+// The warp's 32 rows x 32 words sit in `xs` (row-per-lane layout, stride 33).
+// Write them out transposed: lane L covers rows i*4 + L/8 (i = 0..7) and words
+// (L%8)*4 .. +3, i.e. 8 lanes per 128-byte row segment.  Word w of row r goes to
+// dst_lo(r) + w for w < 16 and to dst_hi(r) + (w - 16) for w >= 16 (two 64-byte
+// segments; for one contiguous 128-byte segment pass dst_hi = dst_lo + 16).
+template <typename RowPtr>
+__device__ __forceinline__ void store_words_transposed(const uint32_t* xs, int lane, int row0, int M, RowPtr dst) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int r = i * 4 + (lane >> 3);
+    const int w = (lane & 7) * 4;
+    if (row0 + r < M) {
+      uint4 v;
+      v.x = xs[r * 33 + w + 0];
+      v.y = xs[r * 33 + w + 1];
+      v.z = xs[r * 33 + w + 2];
+      v.w = xs[r * 33 + w + 3];
+      *reinterpret_cast<uint4*>(dst(r, w)) = v;
+    }
+  }
+}
+
 template <int EPI>
-__device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t taddr, int row, int nb) {
-  const bool in = row < p.M;
-  if constexpr (EPI == EPI_STORE_BF16) {
-    bf16* dst = reinterpret_cast<bf16*>(p.out) + static_cast<int64_t>(row) * p.ld_out + static_cast<int64_t>(nb) * BN;
+__device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t taddr, int mb, int nb, int quarter,
+                                              int lane, uint32_t* xs) {
+  const int row0 = mb * BM + quarter * 32;  // first row of this warp
+  const int row = row0 + lane;              // this thread's row (TMEM lane)
+  if constexpr (EPI == EPI_STORE || EPI == EPI_QKV) {
+    f16* out = reinterpret_cast<f16*>(p.out);
+    const float rs = row_scale(p, row);
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-      uint32_t v[32];
-      tmem_ld32(taddr + c, v);
-      tmem_ld_wait();
-      if (in) {
-        uint4* d4 = reinterpret_cast<uint4*>(dst + c);
+    for (int hh = 0; hh < BN / 128; ++hh) {
+      const int hc = nb * BN + hh * 128;  // first output column of this 128-column head
+      const bool rope = (EPI == EPI_QKV) && hc < p.q_cols + p.k_cols;
+      if (rope) {
+        // per-head RMSNorm (over the 128 columns, of the row-scaled values) then RoPE
+        float ss = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < 128; c += 32) {
+          uint32_t v[32];
+          tmem_ld32(taddr + hh * 128 + c, v);
+          tmem_ld_wait();
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          uint4 w;
-          w.x = pack_bf16x2(__uint_as_float(v[8 * q + 0]), __uint_as_float(v[8 * q + 1]));
-          w.y = pack_bf16x2(__uint_as_float(v[8 * q + 2]), __uint_as_float(v[8 * q + 3]));
-          w.z = pack_bf16x2(__uint_as_float(v[8 * q + 4]), __uint_as_float(v[8 * q + 5]));
-          w.w = pack_bf16x2(__uint_as_float(v[8 * q + 6]), __uint_as_float(v[8 * q + 7]));
-          d4[q] = w;
+          for (int j = 0; j < 32; ++j) ss += __uint_as_float(v[j]) * __uint_as_float(v[j]);
+        }
+        const float inv = rs * rsqrtf(ss * rs * rs * (1.f / 128.f) + p.eps);
+        const bf16* w = hc < p.q_cols ? p.q_norm : p.k_norm;
+        const int pos = row < p.M ? p.tok_pos[row] : 0;
+        const float2* cs = p.rope + static_cast<int64_t>(pos) * 64;
+#pragma unroll 1
+        for (int c = 0; c < 64; c += 32) {
+          uint32_t x1[32], x2[32];
+          tmem_ld32(taddr + hh * 128 + c, x1);
+          tmem_ld32(taddr + hh * 128 + 64 + c, x2);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 32; j += 2) {
+            float y1[2], y2[2];
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const float a = __uint_as_float(x1[j + e]) * inv * __bfloat162float(w[c + j + e]);
+              const float b = __uint_as_float(x2[j + e]) * inv * __bfloat162float(w[64 + c + j + e]);
+              const float2 t = cs[c + j + e];
+              y1[e] = a * t.x - b * t.y;
+              y2[e] = b * t.x + a * t.y;
+            }
+            xs[lane * 33 + j / 2] = pack_f16x2(y1[0], y1[1]);
+            xs[lane * 33 + 16 + j / 2] = pack_f16x2(y2[0], y2[1]);
+          }
+          __syncwarp();
+          store_words_transposed(xs, lane, row0, p.M, [&](int r, int wd) {
+            const int col = hc + c + (wd < 16 ? 2 * wd : 64 + 2 * (wd - 16));
+            return out + static_cast<int64_t>(row0 + r) * p.ld_out + col;
+          });
+          __syncwarp();
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < 128; c += 64) {
+          uint32_t a[32], b[32];
+          tmem_ld32(taddr + hh * 128 + c, a);
+          tmem_ld32(taddr + hh * 128 + c + 32, b);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 32; j += 2) {
+            xs[lane * 33 + j / 2] = pack_f16x2(__uint_as_float(a[j]) * rs, __uint_as_float(a[j + 1]) * rs);
+            xs[lane * 33 + 16 + j / 2] = pack_f16x2(__uint_as_float(b[j]) * rs, __uint_as_float(b[j + 1]) * rs);
+          }
+          __syncwarp();
+          store_words_transposed(xs, lane, row0, p.M, [&](int r, int wd) {
+            return out + static_cast<int64_t>(row0 + r) * p.ld_out + hc + c + 2 * wd;
+          });
+          __syncwarp();
         }
       }
     }
-  } else if constexpr (EPI == EPI_RESID_ADD_F32) {
-    float* dst = reinterpret_cast<float*>(p.out) + static_cast<int64_t>(row) * p.ld_out + static_cast<int64_t>(nb) * BN;
+  } else if constexpr (EPI == EPI_RESID_ADD) {
+    // r += C, then (optionally) the next RMSNorm's operand f16(r * g * rs_pre) and partial sums of r^2.
+    // Lane L owns rows i*4 + L/8 (i = 0..7) and columns (L%8)*4..+3 of each 32-column chunk; the
+    // residual values of chunk c+1 are loaded while chunk c is processed.
+    float* res = reinterpret_cast<float*>(p.out);
+    const int w4 = (lane & 7) * 4;
+    float ss[8], pre[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      ss[i] = 0.f;
+      pre[i] = p.xn_out ? norm_factor(p.ss_pre, p.ss_pre_parts, p, row0 + i * 4 + (lane >> 3)) : 1.f;
+    }
+    auto rrow = [&](int i, int c) {
+      return reinterpret_cast<float4*>(res + static_cast<int64_t>(row0 + i * 4 + (lane >> 3)) * p.ld_out + nb * BN +
+                                       c + w4);
+    };
+    float4 cur[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      cur[i] = (row0 + i * 4 + (lane >> 3) < p.M) ? *rrow(i, 0) : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 1
     for (int c = 0; c < BN; c += 32) {
+      float4 nxt[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        nxt[i] = (c + 32 < BN && row0 + i * 4 + (lane >> 3) < p.M) ? *rrow(i, c + 32) : make_float4(0.f, 0.f, 0.f, 0.f);
       uint32_t v[32];
       tmem_ld32(taddr + c, v);
       tmem_ld_wait();
-      if (in) {
-        float4* d4 = reinterpret_cast<float4*>(dst + c);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          float4 r = d4[q];
-          r.x += __uint_as_float(v[4 * q + 0]);
-          r.y += __uint_as_float(v[4 * q + 1]);
-          r.z += __uint_as_float(v[4 * q + 2]);
-          r.w += __uint_as_float(v[4 * q + 3]);
-          d4[q] = r;
+      for (int j = 0; j < 32; ++j) xs[lane * 33 + j] = v[j];
+      __syncwarp();
+      const int col = nb * BN + c + w4;
+      float4 g4 = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (p.xn_out) {
+        const uint2 gw = *reinterpret_cast<const uint2*>(p.xn_gain + col);
+        const float2 g01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&gw.x));
+        const float2 g23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&gw.y));
+        g4 = make_float4(g01.x, g01.y, g23.x, g23.y);
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int r = i * 4 + (lane >> 3);
+        if (row0 + r < p.M) {
+          float4 x = cur[i];
+          x.x += __uint_as_float(xs[r * 33 + w4 + 0]);
+          x.y += __uint_as_float(xs[r * 33 + w4 + 1]);
+          x.z += __uint_as_float(xs[r * 33 + w4 + 2]);
+          x.w += __uint_as_float(xs[r * 33 + w4 + 3]);
+          *rrow(i, c) = x;
+          if (p.xn_out) {
+            ss[i] += x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w;
+            const float sc = pre[i];
+            uint2 o;
+            o.x = pack_f16x2(x.x * g4.x * sc, x.y * g4.y * sc);
+            o.y = pack_f16x2(x.z * g4.z * sc, x.w * g4.w * sc);
+            *reinterpret_cast<uint2*>(p.xn_out + static_cast<int64_t>(row0 + r) * p.ld_out + col) = o;
+          }
         }
+        cur[i] = nxt[i];
+      }
+      __syncwarp();
+    }
+    if (p.ss_out) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        float t = ss[i];
+        t += __shfl_xor_sync(0xffffffffu, t, 1);
+        t += __shfl_xor_sync(0xffffffffu, t, 2);
+        t += __shfl_xor_sync(0xffffffffu, t, 4);
+        const int r = i * 4 + (lane >> 3);
+        if ((lane & 7) == 0 && row0 + r < p.M) p.ss_out[static_cast<int64_t>(row0 + r) * p.ss_out_parts + nb] = t;
       }
     }
-  } else {  // EPI_SWIGLU_BF16: columns 0..127 gate, 128..255 up of the same 128 outputs
-    bf16* dst = reinterpret_cast<bf16*>(p.out) + static_cast<int64_t>(row) * p.ld_out +
-                static_cast<int64_t>(nb) * (BN / 2);
+  } else {  // EPI_SWIGLU: columns 0..127 gate, 128..255 up of the same 128 outputs
+    f16* out = reinterpret_cast<f16*>(p.out);
+    const float rs = row_scale(p, row);
 #pragma unroll 1
-    for (int c = 0; c < BN / 2; c += 32) {
-      uint32_t g[32], u[32];
-      tmem_ld32(taddr + c, g);
-      tmem_ld32(taddr + BN / 2 + c, u);
-      tmem_ld_wait();
-      if (in) {
-        uint4* d4 = reinterpret_cast<uint4*>(dst + c);
+    for (int c = 0; c < BN / 2; c += 64) {
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          float a[8];
+      for (int half = 0; half < 2; ++half) {
+        uint32_t g[32], u[32];
+        tmem_ld32(taddr + c + 32 * half, g);
+        tmem_ld32(taddr + BN / 2 + c + 32 * half, u);
+        tmem_ld_wait();
 #pragma unroll
-          for (int e = 0; e < 8; ++e)
-            a[e] = silu_f(__uint_as_float(g[8 * q + e])) * __uint_as_float(u[8 * q + e]);
-          uint4 w;
-          w.x = pack_bf16x2(a[0], a[1]);
-          w.y = pack_bf16x2(a[2], a[3]);
-          w.z = pack_bf16x2(a[4], a[5]);
-          w.w = pack_bf16x2(a[6], a[7]);
-          d4[q] = w;
+        for (int j = 0; j < 32; j += 2) {
+          const float a0 = silu_f(__uint_as_float(g[j]) * rs) * (__uint_as_float(u[j]) * rs);
+          const float a1 = silu_f(__uint_as_float(g[j + 1]) * rs) * (__uint_as_float(u[j + 1]) * rs);
+          xs[lane * 33 + 16 * half + j / 2] = pack_f16x2(a0, a1);
         }
       }
+      __syncwarp();
+      store_words_transposed(xs, lane, row0, p.M, [&](int r, int wd) {
+        return out + static_cast<int64_t>(row0 + r) * p.ld_out + nb * (BN / 2) + c + 2 * wd;
+      });
+      __syncwarp();
     }
   }
 }
@@ -132,7 +279,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sA = smem_u32(smem);
   const uint32_t sB = sA + STAGES * A_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint32_t* xpose = reinterpret_cast<uint32_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + XPOSE_BYTES);
   const uint32_t bar0 = smem_u32(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
   auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
@@ -152,7 +300,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull_bar(a), 1);
-      mbar_init(tempty_bar(a), 4);
+      mbar_init(tempty_bar(a), EPI_WARPS);
     }
     mbar_init(drain_bar, 1);
     fence_mbar_init();
@@ -226,7 +374,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const uint64_t bd = umma_desc_sw128(sB + stage * B_BYTES);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)  // +32 bytes along K per step, in 16-byte units
-            umma_bf16(d_tmem, ad + 2 * k, bd + 2 * k, IDESC, (kb | k) != 0);
+            umma_f16(d_tmem, ad + 2 * k, bd + 2 * k, IDESC, (kb | k) != 0);
           umma_commit(empty_bar(stage));
           if (++stage == STAGES) {
             stage = 0;
@@ -242,6 +390,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   } else {
     // ---------------- epilogue warps 2..5 -> TMEM lane quarters 2,3,0,1
     const int quarter = warp & 3;
+    uint32_t* xs = xpose + (warp - 2) * XPOSE_WORDS;
     int local = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x, ++local) {
       int mb, nb;
@@ -251,8 +400,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (!mbar_wait(tfull_bar(acc), acc_phase, p.err, p.timeout_ns)) break;
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
-      const int row = mb * BM + quarter * 32 + lane;
-      epilogue_tile<EPI>(p, taddr, row, nb);
+      epilogue_tile<EPI>(p, taddr, mb, nb, quarter, lane, xs);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty_bar(acc));
@@ -268,33 +416,40 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
+template <int EPI>
+cudaError_t set_smem() {
+  return cudaFuncSetAttribute(k_gemm_tc<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+}
+
 }  // namespace
 
 cudaError_t gemm_setup() {
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(k_gemm_tc<EPI_STORE_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES)))
-    return e;
-  if ((e = cudaFuncSetAttribute(k_gemm_tc<EPI_RESID_ADD_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                SMEM_BYTES)))
-    return e;
-  return cudaFuncSetAttribute(k_gemm_tc<EPI_SWIGLU_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  if ((e = set_smem<EPI_STORE>())) return e;
+  if ((e = set_smem<EPI_RESID_ADD>())) return e;
+  if ((e = set_smem<EPI_SWIGLU>())) return e;
+  return set_smem<EPI_QKV>();
 }
 
-cudaError_t launch_gemm(int epi, const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
-                        int64_t ld_out, int* err, int num_sms, cudaStream_t st) {
-  if (M <= 0) return cudaSuccess;
-  GemmParams p{M, N, K, out, ld_out, err, WAIT_TIMEOUT_NS};
-  const int tiles = ((M + BM - 1) / BM) * (N / BN);
+cudaError_t launch_gemm(int epi, const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& params,
+                        int num_sms, cudaStream_t st) {
+  if (params.M <= 0) return cudaSuccess;
+  GemmParams p = params;
+  p.timeout_ns = WAIT_TIMEOUT_NS;
+  const int tiles = ((p.M + BM - 1) / BM) * (p.N / BN);
   const int grid = tiles < num_sms ? tiles : num_sms;
   switch (epi) {
-    case EPI_STORE_BF16:
-      k_gemm_tc<EPI_STORE_BF16><<<grid, THREADS, SMEM_BYTES, st>>>(tmA, tmB, p);
+    case EPI_STORE:
+      k_gemm_tc<EPI_STORE><<<grid, THREADS, SMEM_BYTES, st>>>(tmA, tmB, p);
       break;
-    case EPI_RESID_ADD_F32:
-      k_gemm_tc<EPI_RESID_ADD_F32><<<grid, THREADS, SMEM_BYTES, st>>>(tmA, tmB, p);
+    case EPI_RESID_ADD:
+      k_gemm_tc<EPI_RESID_ADD><<<grid, THREADS, SMEM_BYTES, st>>>(tmA, tmB, p);
+      break;
+    case EPI_SWIGLU:
+      k_gemm_tc<EPI_SWIGLU><<<grid, THREADS, SMEM_BYTES, st>>>(tmA, tmB, p);
       break;
     default:
-      k_gemm_tc<EPI_SWIGLU_BF16><<<grid, THREADS, SMEM_BYTES, st>>>(tmA, tmB, p);
+      k_gemm_tc<EPI_QKV><<<grid, THREADS, SMEM_BYTES, st>>>(tmA, tmB, p);
       break;
   }
   return cudaGetLastError();

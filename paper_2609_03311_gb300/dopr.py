@@ -23,7 +23,7 @@ STATUS_NAMES = ["OK", "INVALID_ARG", "UNKNOWN_DOC", "INCOMPLETE", "OUT_OF_MEMORY
 (W_EMBED, W_ATTN_NORM, W_Q, W_K, W_V, W_Q_NORM, W_K_NORM, W_O, W_MLP_NORM, W_GATE, W_UP, W_DOWN, W_FINAL_NORM,
  W_SCORE_HEAD) = range(14)
 
-EPI_STORE_BF16, EPI_RESID_ADD_F32, EPI_SWIGLU_BF16 = 0, 1, 2
+EPI_STORE, EPI_RESID_ADD, EPI_SWIGLU = 0, 1, 2
 
 
 class DoprError(RuntimeError):
@@ -232,17 +232,18 @@ def pack_plan(model: Model, store: Store, q_offsets, q_tokens, doc_ids) -> dict:
             "tok_pair": tok_pair[:T]}
 
 
-def gemm(A: torch.Tensor, B: torch.Tensor, epilogue: int = EPI_STORE_BF16, out: torch.Tensor | None = None):
-    """The projection kernel alone: A [M,K] bf16, B [N,K] bf16 (CUDA)."""
+def gemm(A: torch.Tensor, B: torch.Tensor, epilogue: int = EPI_STORE, out: torch.Tensor | None = None):
+    """The projection kernel alone: A [M,K] fp16, B [N,K] fp16 (CUDA)."""
+    assert A.dtype == torch.float16 and B.dtype == torch.float16 and A.is_contiguous() and B.is_contiguous()
     M, K = A.shape
     N = B.shape[0]
     if out is None:
-        if epilogue == EPI_RESID_ADD_F32:
+        if epilogue == EPI_RESID_ADD:
             out = torch.zeros(M, N, dtype=torch.float32, device=A.device)
-        elif epilogue == EPI_SWIGLU_BF16:
-            out = torch.empty(M, N // 2, dtype=torch.bfloat16, device=A.device)
+        elif epilogue == EPI_SWIGLU:
+            out = torch.empty(M, N // 2, dtype=torch.float16, device=A.device)
         else:
-            out = torch.empty(M, N, dtype=torch.bfloat16, device=A.device)
+            out = torch.empty(M, N, dtype=torch.float16, device=A.device)
     st = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
     _check(load().dopr_debug_gemm(M, N, K, _ptr(A), _ptr(B), _ptr(out), epilogue, st))
     return out

@@ -29,19 +29,19 @@ def projections(args):
     g = torch.Generator(device="cuda").manual_seed(0)
 
     def rnd(r, c, std):
-        return (std * torch.randn(r, c, device="cuda", generator=g)).to(torch.bfloat16)
+        return (std * torch.randn(r, c, device="cuda", generator=g)).to(torch.float16)
 
-    cases = [("qkv", rnd(M, H, 1.0), rnd(qkv, H, 0.02), dopr.EPI_STORE_BF16),
-             ("o", rnd(M, o, 1.0), rnd(H, o, 0.02), dopr.EPI_RESID_ADD_F32),
-             ("gate_up", rnd(M, H, 1.0), rnd(2 * F, H, 0.02), dopr.EPI_SWIGLU_BF16),
-             ("down", rnd(M, F, 1.0), rnd(H, F, 0.02), dopr.EPI_RESID_ADD_F32)]
+    cases = [("qkv", rnd(M, H, 1.0), rnd(qkv, H, 0.02), dopr.EPI_STORE),
+             ("o", rnd(M, o, 1.0), rnd(H, o, 0.02), dopr.EPI_RESID_ADD),
+             ("gate_up", rnd(M, H, 1.0), rnd(2 * F, H, 0.02), dopr.EPI_SWIGLU),
+             ("down", rnd(M, F, 1.0), rnd(H, F, 0.02), dopr.EPI_RESID_ADD)]
     out = {}
     for name, A, B, epi in cases:
         res = None
         ms = []
         for _ in range(args.reps):
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            if epi == dopr.EPI_RESID_ADD_F32:
+            if epi == dopr.EPI_RESID_ADD:
                 res = torch.zeros(M, B.shape[0], device="cuda")
             e0.record()
             dopr.gemm(A, B, epi, out=res)

@@ -4,7 +4,7 @@ oracle on identical seeded inputs.
 Bars: |score - oracle| <= 3e-2 absolute; packing plan (pair order, token
 offsets, positions, ids) bit-exact; top-10 order per query identical wherever
 the oracle's adjacent score gap exceeds 0.1.  The projection kernel alone is
-checked against a plain fp32 reference of the same product.
+checked against a plain fp64 reference of the same product.
 """
 import numpy as np
 import pytest
@@ -68,25 +68,25 @@ def _ref_gemm(A, B):
 
 @pytest.mark.parametrize("M,N,K", [(1, 256, 64), (127, 256, 128), (128, 512, 64), (300, 768, 1024),
                                    (1000, 1024, 512), (2085, 1536, 2048)])
-def test_gemm_store_bf16(M, N, K):
+def test_gemm_store_f16(M, N, K):
     g = torch.Generator(device="cuda").manual_seed(M * 7 + N)
-    A = torch.randn(M, K, device="cuda", generator=g).to(torch.bfloat16)
-    B = (0.05 * torch.randn(N, K, device="cuda", generator=g)).to(torch.bfloat16)
-    out = dopr.gemm(A, B, dopr.EPI_STORE_BF16)
+    A = torch.randn(M, K, device="cuda", generator=g).to(torch.float16)
+    B = (0.05 * torch.randn(N, K, device="cuda", generator=g)).to(torch.float16)
+    out = dopr.gemm(A, B, dopr.EPI_STORE)
     torch.cuda.synchronize()
     ref = _ref_gemm(A, B)
     err = (out.double() - ref).abs()
-    assert torch.all(err <= ref.abs() * 2 ** -8 + 1e-4 * ref.abs().max()), float(err.max())
+    assert torch.all(err <= ref.abs() * 2 ** -10 + 1e-4 * ref.abs().max()), float(err.max())
 
 
 @pytest.mark.parametrize("M,N,K", [(5, 256, 64), (333, 512, 512), (1500, 1024, 1536)])
 def test_gemm_residual_add(M, N, K):
     g = torch.Generator(device="cuda").manual_seed(M + 1)
-    A = torch.randn(M, K, device="cuda", generator=g).to(torch.bfloat16)
-    B = (0.05 * torch.randn(N, K, device="cuda", generator=g)).to(torch.bfloat16)
+    A = torch.randn(M, K, device="cuda", generator=g).to(torch.float16)
+    B = (0.05 * torch.randn(N, K, device="cuda", generator=g)).to(torch.float16)
     R = torch.randn(M, N, device="cuda", generator=g)
     ref = _ref_gemm(A, B) + R.double()
-    out = dopr.gemm(A, B, dopr.EPI_RESID_ADD_F32, out=R.clone())
+    out = dopr.gemm(A, B, dopr.EPI_RESID_ADD, out=R.clone())
     torch.cuda.synchronize()
     scale = (A.double().abs() @ B.double().abs().T) + R.double().abs()
     assert torch.all((out.double() - ref).abs() <= 1e-5 * scale + 1e-6)
@@ -95,16 +95,16 @@ def test_gemm_residual_add(M, N, K):
 @pytest.mark.parametrize("M,N,K", [(77, 256, 128), (640, 768, 1024)])
 def test_gemm_swiglu(M, N, K):
     g = torch.Generator(device="cuda").manual_seed(N + K)
-    A = torch.randn(M, K, device="cuda", generator=g).to(torch.bfloat16)
-    B = (0.05 * torch.randn(N, K, device="cuda", generator=g)).to(torch.bfloat16)
-    out = dopr.gemm(A, B, dopr.EPI_SWIGLU_BF16)
+    A = torch.randn(M, K, device="cuda", generator=g).to(torch.float16)
+    B = (0.05 * torch.randn(N, K, device="cuda", generator=g)).to(torch.float16)
+    out = dopr.gemm(A, B, dopr.EPI_SWIGLU)
     torch.cuda.synchronize()
     C = _ref_gemm(A, B)
     blocks = C.view(M, N // 256, 2, 128)
     gate, up = blocks[:, :, 0, :].reshape(M, N // 2), blocks[:, :, 1, :].reshape(M, N // 2)
     ref = torch.nn.functional.silu(gate) * up
     err = (out.double() - ref).abs()
-    assert torch.all(err <= ref.abs() * 2 ** -7 + 1e-4 * ref.abs().max()), float(err.max())
+    assert torch.all(err <= ref.abs() * 2 ** -9 + 1e-4 * ref.abs().max()), float(err.max())
 
 
 # ------------------------------------------------------------ packing plan
@@ -308,8 +308,8 @@ def test_bounded_wait_gives_up_and_context_survives():
     t0 = time.time()
     assert dopr.wait_timeout_probe(200) == dopr.ERR_TIMEOUT
     assert time.time() - t0 < 30
-    A = torch.randn(128, 64, device="cuda").to(torch.bfloat16)
-    B = torch.randn(256, 64, device="cuda").to(torch.bfloat16)
+    A = torch.randn(128, 64, device="cuda").to(torch.float16)
+    B = torch.randn(256, 64, device="cuda").to(torch.float16)
     out = dopr.gemm(A, B)
     torch.cuda.synchronize()
     assert torch.allclose(out.float(), (A.float() @ B.float().T), rtol=1e-2, atol=1e-1)
