@@ -126,7 +126,7 @@ bool kind_is_global(int32_t k) {
 
 void free_workspace(Workspace& w) {
   dev_free(w.r); dev_free(w.xn); dev_free(w.qkv); dev_free(w.o); dev_free(w.act);
-  dev_free(w.ss_e); dev_free(w.ss_a); dev_free(w.ss_m);
+  dev_free(w.ss_e); dev_free(w.ss_a); dev_free(w.ss_m); dev_free(w.r_s); dev_free(w.ss_s);
   dev_free(w.q_off); dev_free(w.q_tok); dev_free(w.doc_ids); dev_free(w.scores);
   dev_free(w.pair_slot); dev_free(w.perm); dev_free(w.sorted_slot); dev_free(w.tok_off);
   dev_free(w.tok_id); dev_free(w.tok_pos); dev_free(w.tok_pair); dev_free(w.doc_count);
@@ -179,6 +179,8 @@ dopr_status alloc_chunk_buffers(Model* m, int cap) {
   STATUS_TRY(dev_alloc(&w.ss_e, (size_t)cap));
   STATUS_TRY(dev_alloc(&w.ss_a, (size_t)cap * (c.hidden / GEMM_BN)));
   STATUS_TRY(dev_alloc(&w.ss_m, (size_t)cap * (c.hidden / GEMM_BN)));
+  STATUS_TRY(dev_alloc(&w.r_s, (size_t)cap * c.hidden));
+  STATUS_TRY(dev_alloc(&w.ss_s, (size_t)cap * (c.hidden / GEMM_BN)));
   STATUS_TRY(dev_alloc(&w.err, 1));
   STATUS_TRY(host_alloc(&w.h_err, 1));
   bool ok = make_tmap_16b_2d(&w.tm_xn, w.xn, c.hidden, cap, (uint64_t)c.hidden * 2, GEMM_BK, GEMM_BM, true, true) &&
@@ -435,7 +437,21 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     base.norm_dim = H;
     base.eps = c.rms_eps;
     base.err = w.err;
+    const int32_t np = s1 - s0;
+    double last_keys = 0.0;  // keys seen by the score-token rows alone
+    for (int32_t sp = s0; sp < s1; ++sp)
+      last_keys += s->slot_m[w.h_sorted_slot[sp]] + (w.h_tok_off[sp + 1] - w.h_tok_off[sp]);
+    const double attn_flops_last = 4.0 * HEAD_DIM * Hq * last_keys;
+    const double attn_bytes_last = np * 2.0 * Hq * HEAD_DIM * 2 + T * 2.0 * Hkv * HEAD_DIM * 2 +
+                                   prefix_rows * Hkv * 2 * HEAD_DIM * 2;
+    const auto op_last = gemm_cost(np, H, m->o_dim, np * H * 10.0);
+    const auto gu_last = gemm_cost(np, 2.0 * F, H, np * F * 2.0);
+    const auto dn_last = gemm_cost(np, H, F, np * H * 8.0);
     for (int l = 0; l < L; ++l) {
+      // In the last layer only the score-token rows reach the score: after the full QKV
+      // projection (every token's key and value is attended to), attention, O and the MLP
+      // run on one compact row per pair.
+      const bool last = l + 1 == L;
       GemmParams pq = base;  // QKV + attention-norm row scale + q/k norm + RoPE
       pq.N = m->qkv_dim;
       pq.K = H;
@@ -470,39 +486,57 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       aa.Hq = Hq;
       aa.Hkv = Hkv;
       aa.mpad_cap = mpad;
+      aa.score_only = last ? 1 : 0;
+      aa.pair_base = s0;
       aa.err = w.err;
-      CUDA_TRY(prof_launch(m, K_ATTENTION, 1, attn_flops, attn_bytes, st,
+      CUDA_TRY(prof_launch(m, K_ATTENTION, 1, last ? attn_flops_last : attn_flops,
+                           last ? attn_bytes_last : attn_bytes, st,
                            [&] { return launch_attention(s->tm_pool, aa, st); }));
+      const float* ss_pre = l == 0 ? w.ss_e : w.ss_a;  // the attention norm of this layer
+      const int ss_pre_parts = l == 0 ? 1 : parts;
+      float* resid = w.r;
+      int rows = Tc;
+      if (last) {
+        CUDA_TRY(prof_launch(m, K_SCORE, 1, 0.0, np * (H * 8.0 + ss_pre_parts * 8.0), st, [&] {
+          return launch_gather_score_rows(w.r, ss_pre, H, ss_pre_parts, w.tok_off, t0, s0, s1, w.r_s, w.ss_s, st);
+        }));
+        ss_pre = w.ss_s;
+        resid = w.r_s;
+        rows = np;
+      }
       GemmParams po = base;  // O projection + residual, emits the MLP norm's operand
+      po.M = rows;
       po.N = H;
       po.K = m->o_dim;
-      po.out = w.r;
+      po.out = resid;
       po.ld_out = H;
       po.xn_out = w.xn;
       po.xn_gain = m->mlp_norm + (size_t)l * H;
       po.ss_out = w.ss_m;
       po.ss_out_parts = parts;
-      po.ss_pre = l == 0 ? w.ss_e : w.ss_a;  // the attention norm of this layer
-      po.ss_pre_parts = l == 0 ? 1 : parts;
-      CUDA_TRY(prof_launch(m, K_GEMM_O, 1, op.first, op.second, st,
+      po.ss_pre = ss_pre;
+      po.ss_pre_parts = ss_pre_parts;
+      CUDA_TRY(prof_launch(m, K_GEMM_O, 1, last ? op_last.first : op.first, last ? op_last.second : op.second, st,
                            [&] { return launch_gemm(EPI_RESID_ADD, w.tm_o, m->tm_o[l], po, sms, st); }));
       GemmParams pg = base;  // gate/up + MLP-norm row scale + SwiGLU
+      pg.M = rows;
       pg.N = 2 * F;
       pg.K = H;
       pg.out = w.act;
       pg.ld_out = F;
       pg.ss_in = w.ss_m;
       pg.ss_parts = parts;
-      pg.ss_pre = po.ss_pre;
-      pg.ss_pre_parts = po.ss_pre_parts;
-      CUDA_TRY(prof_launch(m, K_GEMM_GATE_UP, 1, gu.first, gu.second, st,
-                           [&] { return launch_gemm(EPI_SWIGLU, w.tm_xn, m->tm_gu[l], pg, sms, st); }));
+      pg.ss_pre = ss_pre;
+      pg.ss_pre_parts = ss_pre_parts;
+      CUDA_TRY(prof_launch(m, K_GEMM_GATE_UP, 1, last ? gu_last.first : gu.first, last ? gu_last.second : gu.second,
+                           st, [&] { return launch_gemm(EPI_SWIGLU, w.tm_xn, m->tm_gu[l], pg, sms, st); }));
       GemmParams pd = base;  // down projection + residual, emits the next attention norm's operand
+      pd.M = rows;
       pd.N = H;
       pd.K = F;
-      pd.out = w.r;
+      pd.out = resid;
       pd.ld_out = H;
-      if (l + 1 < L) {
+      if (!last) {
         pd.xn_out = w.xn;
         pd.xn_gain = m->attn_norm + (size_t)(l + 1) * H;
         pd.ss_out = w.ss_a;
@@ -510,12 +544,12 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
         pd.ss_pre = w.ss_m;  // the MLP norm of this layer
         pd.ss_pre_parts = parts;
       }
-      CUDA_TRY(prof_launch(m, K_GEMM_DOWN, 1, dn.first, dn.second, st,
+      CUDA_TRY(prof_launch(m, K_GEMM_DOWN, 1, last ? dn_last.first : dn.first, last ? dn_last.second : dn.second, st,
                            [&] { return launch_gemm(EPI_RESID_ADD, w.tm_act, m->tm_down[l], pd, sms, st); }));
     }
     CUDA_TRY(prof_launch(m, K_SCORE, 1, 4.0 * H * (s1 - s0), (s1 - s0) * (H * 4.0 + 4.0), st, [&] {
-      return launch_score(w.r, H, w.tok_off, t0, s0, s1, w.perm, m->final_norm, m->score_head, c.rms_eps, d_scores,
-                          st);
+      return launch_score(w.r_s, H, w.tok_off, t0, s0, s1, 1, w.perm, m->final_norm, m->score_head, c.rms_eps,
+                          d_scores, st);
     }));
   }
   return DOPR_OK;

@@ -60,6 +60,8 @@ struct Workspace {
   float* ss_e = nullptr;       // [chunk] sum of squares of the embedded rows
   float* ss_a = nullptr;       // [chunk][H/256] partial sums of squares for the attention norm
   float* ss_m = nullptr;       // [chunk][H/256] partial sums of squares for the MLP norm
+  float* r_s = nullptr;        // [chunk][H] score-token rows of the last layer (compact)
+  float* ss_s = nullptr;       // [chunk][H/256] their attention-norm partial sums
   CUtensorMap tm_xn{}, tm_o{}, tm_act{};
   // per call, grown on demand
   int64_t pair_cap = 0, tok_cap = 0, qtok_cap = 0, doc_cap = 0, item_cap = 0;
@@ -175,9 +177,15 @@ cudaError_t launch_embed(const int32_t* tok_id, int T, const bf16* embed, const 
                          f16* xn, float* ss, cudaStream_t st);
 // In place: n bf16 values -> fp16 (saturating at +-65504).
 cudaError_t launch_bf16_to_f16(void* buf, int64_t n, cudaStream_t st);
-cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end,
+// Score head over sorted pairs [p_begin, p_end): the score-token row of pair s is
+// r[tok_off[s+1]-1-tok0], or r[s - p_begin] when `compact` is set.
+cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end, int compact,
                          const int32_t* perm, const bf16* gain, const bf16* head, float eps, float* scores,
                          cudaStream_t st);
+// Compact the score-token rows of sorted pairs [p_begin, p_end): dst_r[i] = r[row(i)] (H floats) and
+// dst_ss[i] = ss[row(i)] (parts floats), row(i) = tok_off[p_begin+i+1]-1-tok0.
+cudaError_t launch_gather_score_rows(const float* r, const float* ss, int H, int parts, const int32_t* tok_off,
+                                     int tok0, int p_begin, int p_end, float* dst_r, float* dst_ss, cudaStream_t st);
 cudaError_t launch_store_transpose(const bf16* k, const bf16* v, int m, int Hkv, bf16* dk, bf16* dv,
                                    cudaStream_t st);
 
@@ -194,6 +202,8 @@ struct AttnArgs {
   const int64_t* slot_row;
   int layer, n_layers, Hq, Hkv;
   int mpad_cap;  // prefix rows reserved in shared memory (multiple of 64)
+  int score_only;  // 1: only each pair's score-token rows, written to out row (pair - pair_base)
+  int pair_base;
   int* err;
 };
 cudaError_t attn_setup();

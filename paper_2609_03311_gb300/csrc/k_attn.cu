@@ -195,10 +195,11 @@ __global__ void __launch_bounds__(THREADS) k_attn(const __grid_constant__ CUtens
     const int tb = a.tok_off[s] - a.tok0;          // first row of the pair in this chunk
     const int T = a.tok_off[s + 1] - a.tok_off[s];  // query tokens + score token
     const int R = T * G;
-    for (int rb = 0; rb * ROWS < R; ++rb) {
-      const int row0 = rb * ROWS + warp * 16;
+    const int rbeg = a.score_only ? (T - 1) * G : 0;  // score-only: just the score token's G rows
+    for (int rb = 0; rbeg + rb * ROWS < R; ++rb) {
+      const int row0 = rbeg + rb * ROWS + warp * 16;
       const bool active = row0 < R;
-      const int jmax = min(T - 1, (rb * ROWS + ROWS - 1) / G);
+      const int jmax = min(T - 1, (rbeg + rb * ROWS + ROWS - 1) / G);
       // ---- Q tile of this warp (16 rows; rows >= R zero-filled)
       if (active) {
 #pragma unroll
@@ -268,7 +269,8 @@ __global__ void __launch_bounds__(THREADS) k_attn(const __grid_constant__ CUtens
           const int row = row0 + (lane >> 2) + hr * 8;
           if (row < R) {
             const int j = row / G, hh = row % G;
-            f16* dst = a.out + static_cast<int64_t>(tb + j) * a.ld_out + (g * G + hh) * HEAD_DIM + (lane & 3) * 2;
+            const int orow = a.score_only ? s - a.pair_base : tb + j;  // compact rows in score-only mode
+            f16* dst = a.out + static_cast<int64_t>(orow) * a.ld_out + (g * G + hh) * HEAD_DIM + (lane & 3) * 2;
             const float inv = hr ? inv1 : inv0;
 #pragma unroll
             for (int dt = 0; dt < 16; ++dt)

@@ -68,11 +68,12 @@ __global__ void k_bf16_to_f16(uint32_t* __restrict__ buf, int64_t n_words) {
 // s = <W[0] - W[1], RMSNorm(r_row) * g>, written to scores[perm[pair]].
 __global__ void __launch_bounds__(ROW_WARPS * 32)
     k_score(const float* __restrict__ r, int H, const int32_t* __restrict__ tok_off, int tok0, int p_begin, int p_end,
-            const int32_t* __restrict__ perm, const bf16* __restrict__ gain, const bf16* __restrict__ head,
-            float eps, float* __restrict__ scores) {
+            int compact, const int32_t* __restrict__ perm, const bf16* __restrict__ gain,
+            const bf16* __restrict__ head, float eps, float* __restrict__ scores) {
   const int s = p_begin + blockIdx.x * ROW_WARPS + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (s >= p_end) return;
-  const float* x = r + static_cast<int64_t>(tok_off[s + 1] - 1 - tok0) * H;
+  const int64_t row = compact ? s - p_begin : tok_off[s + 1] - 1 - tok0;
+  const float* x = r + row * H;
   float ss = 0.f;
   for (int c = lane * 4; c < H; c += 128) {
     const float4 v = *reinterpret_cast<const float4*>(x + c);
@@ -92,6 +93,20 @@ __global__ void __launch_bounds__(ROW_WARPS * 32)
   yes = warp_sum(yes);
   no = warp_sum(no);
   if (lane == 0) scores[perm[s]] = yes - no;
+}
+
+// One warp per pair: copy its score-token row of r (and of the partial sums) to row i.
+__global__ void __launch_bounds__(ROW_WARPS * 32)
+    k_gather_score_rows(const float* __restrict__ r, const float* __restrict__ ss, int H, int parts,
+                        const int32_t* __restrict__ tok_off, int tok0, int p_begin, int p_end,
+                        float* __restrict__ dst_r, float* __restrict__ dst_ss) {
+  const int i = blockIdx.x * ROW_WARPS + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (p_begin + i >= p_end) return;
+  const int64_t row = tok_off[p_begin + i + 1] - 1 - tok0;
+  const float4* src = reinterpret_cast<const float4*>(r + row * H);
+  float4* dst = reinterpret_cast<float4*>(dst_r + static_cast<int64_t>(i) * H);
+  for (int c = lane; c < H / 4; c += 32) dst[c] = src[c];
+  for (int c = lane; c < parts; c += 32) dst_ss[static_cast<int64_t>(i) * parts + c] = ss[row * parts + c];
 }
 
 // [m][Hkv][128] -> [Hkv][m][128] for K and V (16-byte granules).
@@ -142,12 +157,20 @@ cudaError_t launch_bf16_to_f16(void* buf, int64_t n, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end,
+cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end, int compact,
                          const int32_t* perm, const bf16* gain, const bf16* head, float eps, float* scores,
                          cudaStream_t st) {
   if (p_end <= p_begin) return cudaSuccess;
-  k_score<<<blocks_for(p_end - p_begin), ROW_WARPS * 32, 0, st>>>(r, H, tok_off, tok0, p_begin, p_end, perm, gain,
-                                                                  head, eps, scores);
+  k_score<<<blocks_for(p_end - p_begin), ROW_WARPS * 32, 0, st>>>(r, H, tok_off, tok0, p_begin, p_end, compact, perm,
+                                                                  gain, head, eps, scores);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_score_rows(const float* r, const float* ss, int H, int parts, const int32_t* tok_off,
+                                     int tok0, int p_begin, int p_end, float* dst_r, float* dst_ss, cudaStream_t st) {
+  if (p_end <= p_begin) return cudaSuccess;
+  k_gather_score_rows<<<blocks_for(p_end - p_begin), ROW_WARPS * 32, 0, st>>>(r, ss, H, parts, tok_off, tok0, p_begin,
+                                                                              p_end, dst_r, dst_ss);
   return cudaGetLastError();
 }
 

@@ -1,0 +1,53 @@
+"""Full-size parity: each workload at its full model size, scored in the
+launch configuration bench.py times (one batch of 20 queries' candidate
+lists through dopr_score), checked on sampled pairs the oracle computes one
+by one (|score - oracle| <= 3e-2), plus properties that hold at any size
+(finite scores; identical scores when the batch is reversed)."""
+import numpy as np
+import pytest
+import torch
+
+import bench
+from paper_2609_03311_gb300 import dopr, synth
+
+pytestmark = pytest.mark.gpu
+TOL = 3e-2
+
+
+def _sample(pairs, first, n, k, seed):
+    """k pair indices of the batch: the shortest query plus random short-to-median ones."""
+    lens = np.diff(pairs["q_offsets"])[first:first + n]
+    rng = np.random.default_rng(seed)
+    short = np.where(lens <= np.median(lens))[0]
+    pick = [int(np.argmin(lens))] + list(rng.choice(short, size=min(k - 1, len(short)), replace=False))
+    return sorted(set(first + p for p in pick))
+
+
+@pytest.mark.parametrize("workload,n_oracle", [("qwen3-8b-m64", 3), ("qwen3-0.6b", 4), ("qwen3-8b-zipf", 2),
+                                               ("qwen3-4b", 1)])
+def test_full_size_batch_matches_oracle_on_sampled_pairs(workload, n_oracle):
+    wl = synth.WORKLOADS[workload]
+    dev = torch.device("cuda")
+    cfg, model, store, doc_m, w_host = bench.setup(wl, 0, dev, need_host_weights=True)
+    pairs = bench.build_pairs(wl, 0)
+    n = 20 * wl.docs_per_query
+    b = bench.slice_pairs(pairs, 0, n)
+    qo, qt, di = (torch.tensor(b["q_offsets"], device=dev), torch.tensor(b["q_tokens"], device=dev),
+                  torch.tensor(b["doc_ids"], device=dev))
+    got = dopr.score(model, store, qo, qt, di).cpu().numpy()
+    assert np.all(np.isfinite(got))
+    idx = _sample(pairs, 0, n, n_oracle, seed=1)
+    ref, _, _ = bench.oracle_sample(wl, w_host, doc_m, pairs, idx, 0, 1e9, dev)
+    diffs = {p: abs(float(got[p]) - ref[p]) for p in idx}
+    assert max(diffs.values()) <= TOL, diffs
+    if workload == "qwen3-8b-m64":
+        # reversed batch: every pair keeps its score bit for bit
+        rev = np.arange(n)[::-1].copy()
+        lens = np.diff(b["q_offsets"])[rev]
+        qo2 = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+        qt2 = np.concatenate([b["q_tokens"][b["q_offsets"][p]:b["q_offsets"][p + 1]] for p in rev]).astype(np.int32)
+        got2 = dopr.score(model, store, torch.tensor(qo2, device=dev), torch.tensor(qt2, device=dev),
+                          torch.tensor(b["doc_ids"][rev], device=dev)).cpu().numpy()
+        np.testing.assert_array_equal(got2, got[rev])
+    model.close()
+    store.close()
