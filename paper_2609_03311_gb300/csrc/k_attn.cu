@@ -4,15 +4,22 @@
 //
 // One CTA per (work item, kv head).  A work item is a run of consecutive
 // sorted pairs that share one document, so the CTA stages that document's
-// prefix K and V for its kv head (m x 128 bf16 each) into shared memory ONCE
-// with TMA (128-byte swizzle) and reuses it for every query row of every pair
-// in the run.  Rows are (token j, q head of the group) with the G q heads of
-// one kv head interleaved, so a 16-row warp tile covers 16/G tokens x G heads.
-// Per 64-row block the warps sweep the prefix blocks, then stream the pair's
-// own keys 0..j in 64-key chunks (cp.async, zero-filled past the end).
+// prefix K and V for its kv head (m x 128 each) into shared memory ONCE with
+// TMA (128-byte swizzle) and reuses it for every query row of every pair in
+// the run.  Rows are (token j, q head of the group) with the G q heads of one
+// kv head interleaved, so a 16-row warp tile covers 16/G tokens x G heads.
+//
+// Pairs are packed contiguously, so the own keys/values of a batch of
+// consecutive pairs are one block of rows: the CTA loads them once (cp.async)
+// for as many pairs as fit OWN_CAP rows, then the batch's 16-row tiles are
+// dealt round-robin to the warps with no further barriers.  A warp reads its
+// Q tile straight from global memory into mma fragments, sweeps the prefix in
+// 32-key blocks, then its own causal keys in 16-key blocks, with the online
+// (running max / running sum) softmax.  Pairs longer
+// than OWN_CAP stream their own keys in OWN_CAP chunks per 64-row group.
 // Scores and P.V use warp-level fp16 mma with fp32 accumulation (the stored
-// bf16 prefix is widened to fp16 in shared memory after it lands); the softmax
-// is the online (running max / running sum) form with quad shuffles.
+// bf16 prefix is widened to fp16 in shared memory after it lands); row maxima
+// and sums use quad shuffles.
 #include <math.h>
 
 #include "device_common.cuh"
@@ -23,48 +30,55 @@ namespace {
 
 constexpr int WARPS = 4;
 constexpr int THREADS = WARPS * 32;
-constexpr int ROWS = WARPS * 16;   // rows per row block
-constexpr int KEYS = 64;           // keys per block
 constexpr int ROW_BYTES = HEAD_DIM * 2;
-constexpr int BOX_BYTES = 64 * 128;      // TMA box: 64 rows x 64 elements
-constexpr int OWN_BYTES = KEYS * ROW_BYTES;  // own K (or V) chunk
-constexpr int Q_BYTES = 16 * ROW_BYTES;      // per-warp Q tile
+constexpr int BOX_BYTES = 64 * 128;          // TMA box: 64 rows x 64 elements
+constexpr int OWN_CAP = 64;                  // own key rows resident at once
+constexpr int OWN_ROWS = OWN_CAP + 16;       // + zeroed tail read by the last 16-key block
+constexpr int OWN_BYTES = OWN_ROWS * ROW_BYTES;
+constexpr int MAX_BATCH = 32;                // pairs per resident batch
+#ifndef DOPR_ATTN_MIN_BLOCKS
+#define DOPR_ATTN_MIN_BLOCKS 2                 // resident CTAs per SM the register budget targets
+#endif
 
-// Byte offset of (row r, 16-byte chunk c) in a tile of 64-row boxes, each box
+// Prefix tile: byte offset of (row r, 16-byte chunk c) in 64-row boxes, each
 // split into two 64-element halves, 128-byte swizzled (what TMA writes).
-__device__ __forceinline__ uint32_t off64(int r, int c) {
+__device__ __forceinline__ uint32_t off_pre(int r, int c) {
   return static_cast<uint32_t>((((r >> 6) * 2 + (c >> 3)) * 64 + (r & 63)) * 128 + (((c & 7) ^ (r & 7)) << 4));
 }
-// Same layout for a 16-row tile.
-__device__ __forceinline__ uint32_t off16(int r, int c) {
-  return static_cast<uint32_t>(((c >> 3) * 16 + r) * 128 + (((c & 7) ^ (r & 7)) << 4));
+// Own-key tile: 256-byte rows, 16-byte chunks XOR-swizzled by the row (conflict-free ldmatrix).
+__device__ __forceinline__ uint32_t off_own(int r, int c) {
+  return static_cast<uint32_t>(r * ROW_BYTES + ((c ^ (r & 7)) << 4));
 }
 
-// One 64-key block for one warp's 16 rows.  kbase/vbase point at a 64-row box
-// pair of the K and V tiles.  Keys kk >= n_valid are masked; with CAUSAL a key
-// kk is visible to a row of token j only if key0 + kk <= j.
-template <bool CAUSAL>
-__device__ __forceinline__ void attend_block(uint32_t kbase, uint32_t vbase, int lane, const uint32_t (&qf)[8][4],
-                                             float (&o)[16][4], float (&mrow)[2], float (&lrow)[2], int n_valid,
-                                             int key0, const int (&jr)[2], float scale_log2) {
-  float s[8][4];
+struct TileState {
+  float o[16][4];
+  float mrow[2], lrow[2];
+};
+
+// One block of NT*8 keys for one warp's 16 rows.  Keys kk >= n_valid are
+// masked; with CAUSAL key kk is visible to a row of token j only if key0 + kk <= j.
+template <int NT, bool CAUSAL, bool PREFIX>
+__device__ __forceinline__ void attend(uint32_t kt, uint32_t vt, int kbase, int lane, const uint32_t (&qf)[8][4],
+                                       TileState& st, int n_valid, int key0, const int (&jr)[2], float scale_log2) {
+  auto off = [](int r, int c) { return PREFIX ? off_pre(r, c) : off_own(r, c); };
+  float s[NT][4];
 #pragma unroll
-  for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+  for (int nt = 0; nt < NT; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
 #pragma unroll
-    for (int np = 0; np < 4; ++np) {
-      const int key = np * 16 + (lane & 7) + ((lane >> 4) << 3);
+    for (int np = 0; np < NT / 2; ++np) {
+      const int key = kbase + np * 16 + (lane & 7) + ((lane >> 4) << 3);
       const int c = 2 * ks + ((lane >> 3) & 1);
       uint32_t b0, b1, b2, b3;
-      ldmatrix_x4(kbase + off64(key, c), b0, b1, b2, b3);
+      ldmatrix_x4(kt + off(key, c), b0, b1, b2, b3);
       mma_f16_16816(s[2 * np], qf[ks], b0, b1);
       mma_f16_16816(s[2 * np + 1], qf[ks], b2, b3);
     }
   }
   float mx[2] = {-INFINITY, -INFINITY};
 #pragma unroll
-  for (int nt = 0; nt < 8; ++nt)
+  for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       const int kk = nt * 8 + (lane & 3) * 2 + (e & 1);
@@ -79,57 +93,133 @@ __device__ __forceinline__ void attend_block(uint32_t kbase, uint32_t vbase, int
   for (int i = 0; i < 2; ++i) {
     mx[i] = fmaxf(mx[i], __shfl_xor_sync(0xffffffffu, mx[i], 1));
     mx[i] = fmaxf(mx[i], __shfl_xor_sync(0xffffffffu, mx[i], 2));
-    const float mnew = fmaxf(mrow[i], mx[i]);
+    const float mnew = fmaxf(st.mrow[i], mx[i]);
     base[i] = (mnew == -INFINITY) ? 0.f : mnew;
-    alpha[i] = exp2f(mrow[i] - base[i]);
-    mrow[i] = mnew;
+    alpha[i] = exp2f(st.mrow[i] - base[i]);
+    st.mrow[i] = mnew;
   }
   float rs[2] = {0.f, 0.f};
 #pragma unroll
-  for (int nt = 0; nt < 8; ++nt)
+  for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       const float p = exp2f(s[nt][e] - base[e >> 1]);
       s[nt][e] = p;
       rs[e >> 1] += p;
     }
-  lrow[0] = lrow[0] * alpha[0] + rs[0];
-  lrow[1] = lrow[1] * alpha[1] + rs[1];
+  st.lrow[0] = st.lrow[0] * alpha[0] + rs[0];
+  st.lrow[1] = st.lrow[1] * alpha[1] + rs[1];
 #pragma unroll
   for (int dt = 0; dt < 16; ++dt) {
-    o[dt][0] *= alpha[0];
-    o[dt][1] *= alpha[0];
-    o[dt][2] *= alpha[1];
-    o[dt][3] *= alpha[1];
+    st.o[dt][0] *= alpha[0];
+    st.o[dt][1] *= alpha[0];
+    st.o[dt][2] *= alpha[1];
+    st.o[dt][3] *= alpha[1];
   }
 #pragma unroll
-  for (int kk = 0; kk < 4; ++kk) {
-    uint32_t a[4];
-    a[0] = pack_f16x2(s[2 * kk][0], s[2 * kk][1]);
-    a[1] = pack_f16x2(s[2 * kk][2], s[2 * kk][3]);
-    a[2] = pack_f16x2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-    a[3] = pack_f16x2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
+  for (int kk = 0; kk < NT / 2; ++kk) {
+    uint32_t pa[4];
+    pa[0] = pack_f16x2(s[2 * kk][0], s[2 * kk][1]);
+    pa[1] = pack_f16x2(s[2 * kk][2], s[2 * kk][3]);
+    pa[2] = pack_f16x2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
+    pa[3] = pack_f16x2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
 #pragma unroll
     for (int dp = 0; dp < 8; ++dp) {
-      const int key = kk * 16 + (lane & 7) + (((lane >> 3) & 1) << 3);
+      const int key = kbase + kk * 16 + (lane & 7) + (((lane >> 3) & 1) << 3);
       const int c = 2 * dp + (lane >> 4);
       uint32_t b0, b1, b2, b3;
-      ldmatrix_x4_trans(vbase + off64(key, c), b0, b1, b2, b3);
-      mma_f16_16816(o[2 * dp], a, b0, b1);
-      mma_f16_16816(o[2 * dp + 1], a, b2, b3);
+      ldmatrix_x4_trans(vt + off(key, c), b0, b1, b2, b3);
+      mma_f16_16816(st.o[2 * dp], pa, b0, b1);
+      mma_f16_16816(st.o[2 * dp + 1], pa, b2, b3);
     }
   }
 }
 
-__global__ void __launch_bounds__(THREADS) k_attn(const __grid_constant__ CUtensorMap tm_pool, AttnArgs a) {
+struct PairGeom {
+  int tb;  // first row of the pair in this chunk
+  int T;   // tokens (query + score token)
+  int R;   // rows = T * G
+};
+
+// Q fragments of rows row0..row0+15 straight from global memory (rows >= R read as 0).
+__device__ __forceinline__ void load_q(const AttnArgs& a, const PairGeom& pg, int g, int G, int row0, int lane,
+                                       uint32_t (&qf)[8][4]) {
+  const int ra = row0 + (lane >> 2), rb = ra + 8;
+  const uint32_t* qa = nullptr;
+  const uint32_t* qb = nullptr;
+  if (ra < pg.R)
+    qa = reinterpret_cast<const uint32_t*>(a.qkv + static_cast<int64_t>(pg.tb + ra / G) * a.ld_qkv +
+                                           (g * G + ra % G) * HEAD_DIM);
+  if (rb < pg.R)
+    qb = reinterpret_cast<const uint32_t*>(a.qkv + static_cast<int64_t>(pg.tb + rb / G) * a.ld_qkv +
+                                           (g * G + rb % G) * HEAD_DIM);
+  const int t = lane & 3;
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    const int w = ks * 8 + t;  // 32-bit word index of columns 16ks + 2t
+    qf[ks][0] = qa ? __ldg(qa + w) : 0u;
+    qf[ks][1] = qb ? __ldg(qb + w) : 0u;
+    qf[ks][2] = qa ? __ldg(qa + w + 4) : 0u;
+    qf[ks][3] = qb ? __ldg(qb + w + 4) : 0u;
+  }
+}
+
+__device__ __forceinline__ void init_state(TileState& st) {
+#pragma unroll
+  for (int dt = 0; dt < 16; ++dt) st.o[dt][0] = st.o[dt][1] = st.o[dt][2] = st.o[dt][3] = 0.f;
+  st.mrow[0] = st.mrow[1] = -INFINITY;
+  st.lrow[0] = st.lrow[1] = 0.f;
+}
+
+// Normalise and store the tile's rows < R (compact row per pair in score-only mode).
+__device__ __forceinline__ void store_tile(const AttnArgs& a, const PairGeom& pg, int s, int g, int G, int row0,
+                                           int lane, TileState& st) {
+  float l0 = st.lrow[0], l1 = st.lrow[1];
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+  const float inv0 = l0 > 0.f ? 1.f / l0 : 0.f, inv1 = l1 > 0.f ? 1.f / l1 : 0.f;
+#pragma unroll
+  for (int hr = 0; hr < 2; ++hr) {
+    const int row = row0 + (lane >> 2) + hr * 8;
+    if (row < pg.R) {
+      const int j = row / G, hh = row % G;
+      const int orow = a.score_only ? s - a.pair_base : pg.tb + j;
+      f16* dst = a.out + static_cast<int64_t>(orow) * a.ld_out + (g * G + hh) * HEAD_DIM + (lane & 3) * 2;
+      const float inv = hr ? inv1 : inv0;
+#pragma unroll
+      for (int dt = 0; dt < 16; ++dt)
+        *reinterpret_cast<uint32_t*>(dst + dt * 8) = pack_f16x2(st.o[dt][2 * hr] * inv, st.o[dt][2 * hr + 1] * inv);
+    }
+  }
+}
+
+// Own keys/values of chunk rows [row_begin, row_begin + count) into own-buffer
+// rows 0..count-1; rows count .. count+15 are zeroed.  All threads take part.
+__device__ __forceinline__ void load_own(const AttnArgs& a, int g, uint32_t sOK, uint32_t sOV, int row_begin,
+                                         int count, int tid) {
+  const int kcol = (a.Hq + g) * HEAD_DIM;
+  const int vcol = (a.Hq + a.Hkv + g) * HEAD_DIM;
+  const int rows = min(OWN_ROWS, count + 16);
+  for (int idx = tid; idx < rows * 32; idx += THREADS) {
+    const int kv = idx & 1, rc = idx >> 1, r = rc >> 4, c = rc & 15;
+    const bool ok = r < count;
+    const f16* src = a.qkv + static_cast<int64_t>(row_begin + (ok ? r : 0)) * a.ld_qkv + (kv ? vcol : kcol) + c * 8;
+    cp_async16((kv ? sOV : sOK) + off_own(r, c), src, ok);
+  }
+  cp_async_commit();
+  cp_async_wait_all();
+}
+
+__global__ void __launch_bounds__(THREADS, DOPR_ATTN_MIN_BLOCKS) k_attn(const __grid_constant__ CUtensorMap tm_pool, AttnArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sPK = smem_u32(smem);
   const uint32_t sPV = sPK + a.mpad_cap * ROW_BYTES;
   const uint32_t sOK = sPV + a.mpad_cap * ROW_BYTES;
   const uint32_t sOV = sOK + OWN_BYTES;
-  const uint32_t sQ0 = sOV + OWN_BYTES;
-  const uint32_t bar = sQ0 + WARPS * Q_BYTES;
+  const uint32_t bar = sOV + OWN_BYTES;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const AttnItem item = a.items[blockIdx.x];
@@ -169,8 +259,8 @@ __global__ void __launch_bounds__(THREADS) k_attn(const __grid_constant__ CUtens
     uint8_t* gv = smem + a.mpad_cap * ROW_BYTES;
     for (int i = tid; i < nbox * 64 * 16; i += THREADS) {
       const int r = i / 16, c = i % 16;
-      uint4* pk = reinterpret_cast<uint4*>(gk + off64(r, c));
-      uint4* pv = reinterpret_cast<uint4*>(gv + off64(r, c));
+      uint4* pk = reinterpret_cast<uint4*>(gk + off_pre(r, c));
+      uint4* pv = reinterpret_cast<uint4*>(gv + off_pre(r, c));
       if (r >= m) {
         *pk = make_uint4(0, 0, 0, 0);
         *pv = make_uint4(0, 0, 0, 0);
@@ -182,108 +272,90 @@ __global__ void __launch_bounds__(THREADS) k_attn(const __grid_constant__ CUtens
         *pv = y;
       }
     }
-    __syncthreads();
+    // (the barrier before the first own-key load orders these writes)
   }
 
-  const f16* qkv = a.qkv;
-  const int ld = a.ld_qkv;
-  const int kcol = (a.Hq + g) * HEAD_DIM;
-  const int vcol = (a.Hq + a.Hkv + g) * HEAD_DIM;
-  const uint32_t sQ = sQ0 + warp * Q_BYTES;
+  auto geom = [&](int s) {
+    PairGeom pg;
+    pg.tb = a.tok_off[s] - a.tok0;
+    pg.T = a.tok_off[s + 1] - a.tok_off[s];
+    pg.R = pg.T * G;
+    return pg;
+  };
+  auto prefix_pass = [&](const uint32_t (&qf)[8][4], TileState& st, const int (&jr)[2]) {
+    for (int k0 = 0; k0 < m; k0 += 32)
+      attend<4, false, true>(sPK, sPV, k0, lane, qf, st, min(32, m - k0), 0, jr, scale_log2);
+  };
 
-  for (int s = item.pair_begin; s < item.pair_end; ++s) {
-    const int tb = a.tok_off[s] - a.tok0;          // first row of the pair in this chunk
-    const int T = a.tok_off[s + 1] - a.tok_off[s];  // query tokens + score token
-    const int R = T * G;
-    const int rbeg = a.score_only ? (T - 1) * G : 0;  // score-only: just the score token's G rows
-    for (int rb = 0; rbeg + rb * ROWS < R; ++rb) {
-      const int row0 = rbeg + rb * ROWS + warp * 16;
-      const bool active = row0 < R;
-      const int jmax = min(T - 1, (rbeg + rb * ROWS + ROWS - 1) / G);
-      // ---- Q tile of this warp (16 rows; rows >= R zero-filled)
-      if (active) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int idx = lane + i * 32, r = idx >> 4, c = idx & 15;
-          const int row = row0 + r;
-          const bool ok = row < R;
-          const int j = ok ? row / G : 0, hh = ok ? row % G : 0;
-          const f16* src = qkv + static_cast<int64_t>(tb + j) * ld + (g * G + hh) * HEAD_DIM + c * 8;
-          cp_async16(sQ + off16(r, c), src, ok);
+  int s = item.pair_begin;
+  while (s < item.pair_end) {
+    const PairGeom p0 = geom(s);
+    if (p0.T <= OWN_CAP) {
+      // ---- resident batch: pairs [s, e) whose own rows fit OWN_CAP together
+      int e = s + 1, rows = p0.T;
+      while (e < item.pair_end && e - s < MAX_BATCH) {
+        const int t = a.tok_off[e + 1] - a.tok_off[e];
+        if (rows + t > OWN_CAP) break;
+        rows += t;
+        ++e;
+      }
+      __syncthreads();  // previous users of the own buffer are done
+      load_own(a, g, sOK, sOV, p0.tb, rows, tid);
+      __syncthreads();
+      int tile = 0;
+      for (int sp = s; sp < e; ++sp) {
+        const PairGeom pg = geom(sp);
+        const int rbeg = a.score_only ? (pg.T - 1) * G : 0;
+        const int own_base = pg.tb - p0.tb;
+        for (int row0 = rbeg; row0 < pg.R; row0 += 16, ++tile) {
+          if ((tile % WARPS) != warp) continue;
+          uint32_t qf[8][4];
+          load_q(a, pg, g, G, row0, lane, qf);
+          TileState st;
+          init_state(st);
+          const int jr[2] = {(row0 + (lane >> 2)) / G, (row0 + (lane >> 2) + 8) / G};
+          prefix_pass(qf, st, jr);
+          const int jmax = min(pg.T - 1, (row0 + 15) / G);
+          for (int k0 = 0; k0 <= jmax; k0 += 16)
+            attend<2, true, false>(sOK, sOV, own_base + k0, lane, qf, st, 16, k0, jr, scale_log2);
+          store_tile(a, pg, sp, g, G, row0, lane, st);
         }
       }
-      cp_async_commit();
-      cp_async_wait_all();
-      __syncwarp();
-      uint32_t qf[8][4];
-      float o[16][4];
-      float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
-      int jr[2];
-      {
-        const int r0 = row0 + (lane >> 2);
-        jr[0] = r0 / G;
-        jr[1] = (r0 + 8) / G;
-      }
-#pragma unroll
-      for (int dt = 0; dt < 16; ++dt) o[dt][0] = o[dt][1] = o[dt][2] = o[dt][3] = 0.f;
-      if (active) {
-#pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-          const int r = (lane & 7) + (((lane >> 3) & 1) << 3);
-          const int c = 2 * ks + (lane >> 4);
-          ldmatrix_x4(sQ + off16(r, c), qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3]);
+      s = e;
+    } else {
+      // ---- long pair: 64-row groups, own keys streamed in OWN_CAP chunks
+      const PairGeom pg = p0;
+      const int rbeg = a.score_only ? (pg.T - 1) * G : 0;
+      for (int rg = rbeg; rg < pg.R; rg += WARPS * 16) {
+        const int row0 = rg + warp * 16;
+        const bool active = row0 < pg.R;
+        uint32_t qf[8][4];
+        TileState st;
+        init_state(st);
+        const int jr[2] = {(row0 + (lane >> 2)) / G, (row0 + (lane >> 2) + 8) / G};
+        if (active) {
+          load_q(a, pg, g, G, row0, lane, qf);
+          prefix_pass(qf, st, jr);
         }
-        // ---- prefix keys: visible to every online token
-        for (int kb = 0; kb < nbox; ++kb)
-          attend_block<false>(sPK + kb * 2 * BOX_BYTES, sPV + kb * 2 * BOX_BYTES, lane, qf, o, mrow, lrow,
-                              min(KEYS, m - kb * KEYS), 0, jr, scale_log2);
-      }
-      // ---- own keys 0..jmax in chunks of 64, causal
-      for (int c0 = 0; c0 <= jmax; c0 += KEYS) {
-        __syncthreads();  // previous chunk fully consumed
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int idx = tid + i * THREADS;  // 0 .. 2047
-          const int kv = idx >> 10, rem = idx & 1023, key = rem >> 4, c = rem & 15;
-          const bool ok = c0 + key <= jmax;
-          const int row = tb + (ok ? c0 + key : 0);
-          const f16* src = qkv + static_cast<int64_t>(row) * ld + (kv ? vcol : kcol) + c * 8;
-          cp_async16((kv ? sOV : sOK) + off64(key, c), src, ok);
+        const int jmax_g = min(pg.T - 1, (rg + WARPS * 16 - 1) / G);
+        const int jmax = min(pg.T - 1, (row0 + 15) / G);
+        for (int c0 = 0; c0 <= jmax_g; c0 += OWN_CAP) {
+          __syncthreads();
+          load_own(a, g, sOK, sOV, pg.tb + c0, min(OWN_CAP, jmax_g + 1 - c0), tid);
+          __syncthreads();
+          if (active)
+            for (int k0 = c0; k0 <= min(jmax, c0 + OWN_CAP - 1); k0 += 16)
+              attend<2, true, false>(sOK, sOV, k0 - c0, lane, qf, st, 16, k0, jr, scale_log2);
         }
-        cp_async_commit();
-        cp_async_wait_all();
-        __syncthreads();
-        if (active)
-          attend_block<true>(sOK, sOV, lane, qf, o, mrow, lrow, min(KEYS, jmax + 1 - c0), c0, jr, scale_log2);
+        if (active) store_tile(a, pg, s, g, G, row0, lane, st);
       }
-      // ---- normalise and store rows < R
-      if (active) {
-        float l0 = lrow[0], l1 = lrow[1];
-        l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-        l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-        l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-        l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-        const float inv0 = l0 > 0.f ? 1.f / l0 : 0.f, inv1 = l1 > 0.f ? 1.f / l1 : 0.f;
-#pragma unroll
-        for (int hr = 0; hr < 2; ++hr) {
-          const int row = row0 + (lane >> 2) + hr * 8;
-          if (row < R) {
-            const int j = row / G, hh = row % G;
-            const int orow = a.score_only ? s - a.pair_base : tb + j;  // compact rows in score-only mode
-            f16* dst = a.out + static_cast<int64_t>(orow) * a.ld_out + (g * G + hh) * HEAD_DIM + (lane & 3) * 2;
-            const float inv = hr ? inv1 : inv0;
-#pragma unroll
-            for (int dt = 0; dt < 16; ++dt)
-              *reinterpret_cast<uint32_t*>(dst + dt * 8) = pack_f16x2(o[dt][2 * hr] * inv, o[dt][2 * hr + 1] * inv);
-          }
-        }
-      }
+      ++s;
     }
   }
 }
 
 inline size_t attn_smem_bytes(int mpad_cap) {
-  return 1024 + 2 * static_cast<size_t>(mpad_cap) * ROW_BYTES + 2 * OWN_BYTES + WARPS * Q_BYTES + 64;
+  return 1024 + 2 * static_cast<size_t>(mpad_cap) * ROW_BYTES + 2 * OWN_BYTES + 64;
 }
 
 }  // namespace
