@@ -242,7 +242,7 @@ DOPR_API dopr_status dopr_pack_order_noalloc(const dopr_store *store, int32_t n_
 
 /*
  * Per-kernel accounting, for measurement.  Every dopr_score call counts its
- * kernel launches per kernel family (pack, embed_norm, gemm_qkv, qknorm_rope,
+ * kernel launches per kernel family (pack, embed, gemm_qkv, qknorm_rope,
  * attention, gemm_o, rmsnorm, gemm_gate_up, gemm_down, score) together with
  * the algorithmic floating-point operations and device-memory bytes of those
  * launches (the minimum the operation needs: each input read once, each output

@@ -137,6 +137,21 @@ def test_scores_match_oracle_ragged(shape):
     assert np.max(np.abs(got - ref)) <= TOL, np.max(np.abs(got - ref))
 
 
+@pytest.mark.parametrize("shape", [SMALL_G2, SMALL_G4], ids=["G2", "G4"])
+@pytest.mark.parametrize("doc_m", [{0: 0, 1: 1, 2: 17, 3: 63, 4: 64}, {0: 65, 1: 100, 2: 128, 3: 3}],
+                         ids=["mpad64", "mpad128"])
+def test_scores_match_oracle_short_prefixes_long_queries(shape, doc_m):
+    # Prefixes of at most 128 rows with queries up to 160 tokens: pairs whose
+    # own keys fit the attention kernel's resident buffer share batches, the
+    # longer ones stream their keys in chunks; both must match the oracle.
+    rig = Rig(shape, doc_m, seed=15)
+    pairs = synth.random_pairs(48, len(doc_m), 0, 160, shape.vocab, seed=15)
+    got = rig.score(pairs)
+    ref = rig.oracle(pairs)
+    assert np.all(np.isfinite(got))
+    assert np.max(np.abs(got - ref)) <= TOL, np.max(np.abs(got - ref))
+
+
 def test_empty_queries_and_empty_prefix():
     rig = Rig(SMALL_G2, {0: 0, 1: 8}, seed=6)
     pairs = {"q_offsets": np.array([0, 0, 0, 3, 3], np.int32), "q_tokens": np.array([5, 6, 7], np.int32),
