@@ -177,10 +177,11 @@ dopr_status alloc_chunk_buffers(Model* m, int cap) {
   STATUS_TRY(dev_alloc(&w.o, (size_t)cap * m->o_dim));
   STATUS_TRY(dev_alloc(&w.act, (size_t)cap * c.ffn));
   STATUS_TRY(dev_alloc(&w.ss_e, (size_t)cap));
-  STATUS_TRY(dev_alloc(&w.ss_a, (size_t)cap * (c.hidden / GEMM_BN)));
-  STATUS_TRY(dev_alloc(&w.ss_m, (size_t)cap * (c.hidden / GEMM_BN)));
+  const size_t parts = (size_t)(c.hidden / GEMM_BN) * GEMM_SS_PER_TILE;
+  STATUS_TRY(dev_alloc(&w.ss_a, (size_t)cap * parts));
+  STATUS_TRY(dev_alloc(&w.ss_m, (size_t)cap * parts));
   STATUS_TRY(dev_alloc(&w.r_s, (size_t)cap * c.hidden));
-  STATUS_TRY(dev_alloc(&w.ss_s, (size_t)cap * (c.hidden / GEMM_BN)));
+  STATUS_TRY(dev_alloc(&w.ss_s, (size_t)cap * parts));
   STATUS_TRY(dev_alloc(&w.err, 1));
   STATUS_TRY(host_alloc(&w.h_err, 1));
   bool ok = make_tmap_16b_2d(&w.tm_xn, w.xn, c.hidden, cap, (uint64_t)c.hidden * 2, GEMM_BK, GEMM_BM, true, true) &&
@@ -405,7 +406,7 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
   Workspace& w = m->ws;
   const auto& c = m->cfg;
   const int H = c.hidden, F = c.ffn, L = c.n_layers, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
-  const int parts = H / GEMM_BN;  // partial sums of squares per row from a residual epilogue
+  const int parts = H / GEMM_BN * GEMM_SS_PER_TILE;  // partial sums of squares per row from a residual epilogue
   const int mpad = ((s->max_m + 63) / 64) * 64;
   const int sms = m->num_sms;
   auto gemm_cost = [](double M, double N, double K, double out_bytes) {

@@ -58,10 +58,10 @@ struct Workspace {
   f16* o = nullptr;            // [chunk][Hq*128] attention output
   f16* act = nullptr;          // [chunk][F] SwiGLU output
   float* ss_e = nullptr;       // [chunk] sum of squares of the embedded rows
-  float* ss_a = nullptr;       // [chunk][H/256] partial sums of squares for the attention norm
-  float* ss_m = nullptr;       // [chunk][H/256] partial sums of squares for the MLP norm
+  float* ss_a = nullptr;       // [chunk][2H/256] partial sums of squares for the attention norm
+  float* ss_m = nullptr;       // [chunk][2H/256] partial sums of squares for the MLP norm
   float* r_s = nullptr;        // [chunk][H] score-token rows of the last layer (compact)
-  float* ss_s = nullptr;       // [chunk][H/256] their attention-norm partial sums
+  float* ss_s = nullptr;       // [chunk][2H/256] their attention-norm partial sums
   CUtensorMap tm_xn{}, tm_o{}, tm_act{};
   // per call, grown on demand
   int64_t pair_cap = 0, tok_cap = 0, qtok_cap = 0, doc_cap = 0, item_cap = 0;
@@ -138,6 +138,7 @@ bool make_tmap_16b_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_
 // GEMM epilogues.
 enum GemmEpi : int { EPI_STORE = 0, EPI_RESID_ADD = 1, EPI_SWIGLU = 2, EPI_QKV = 3 };
 constexpr int GEMM_BM = 128, GEMM_BN = 256, GEMM_BK = 64;
+constexpr int GEMM_SS_PER_TILE = 2;  // partial sums of squares a residual epilogue writes per row and n-tile
 struct GemmParams {
   int M, N, K;
   void* out;          // fp16 [M][ld_out] (store, QKV, SwiGLU: ld_out = N/2) or fp32 residual [M][ld_out]

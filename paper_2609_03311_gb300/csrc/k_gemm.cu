@@ -8,8 +8,9 @@
 //   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and one
 //               elected thread issues tcgen05.mma (M=128, N=256, K=16) per k-step,
 //               committing stage releases and accumulator-ready barriers;
-//   warps 2..5  epilogue: tcgen05.ld the finished accumulator (one TMEM lane quarter
-//               = 32 rows per warp, one row per thread), apply the epilogue in that
+//   warps 2..9  epilogue: tcgen05.ld the finished accumulator (one TMEM lane quarter
+//               = 32 rows per warp, one row per thread; two warps per quarter, each
+//               taking half of the tile's 256 columns), apply the epilogue in that
 //               row-per-thread layout, then transpose 32x32-word chunks through
 //               padded shared memory so every global access is a 128-byte row
 //               segment written by 8 consecutive lanes; finally release the
@@ -25,7 +26,8 @@
 //   tile, the partial sum of r'^2.  The consuming GEMM sums those partials
 //   (in a fixed order) and scales its accumulator rows by rs / rs_pre.
 //   QKV epilogue: row scale, then per 128-column q/k head RMSNorm with the
-//   q/k gain and rotate-half RoPE at the token's position (pairs i, i+64).
+//   q/k gain and rotate-half RoPE at the token's position (pairs i, i+64),
+//   the rotation applied in the transposed layout so RoPE-table reads coalesce.
 //   SwiGLU epilogue: silu(rs * gate) * (rs * up).
 // Every barrier wait is bounded (DEV_ERR_TIMEOUT) and the kernel always drains
 // its own copies and MMAs and frees TMEM before returning.
@@ -41,8 +43,8 @@ constexpr int A_BYTES = BM * BK * 2;  // 16 KiB
 constexpr int B_BYTES = BN * BK * 2;  // 32 KiB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 2 * BN;     // two accumulators
-constexpr int THREADS = 192;
-constexpr int EPI_WARPS = 4;
+constexpr int THREADS = 320;
+constexpr int EPI_WARPS = 8;
 constexpr int GROUP_M = 16;
 constexpr int XPOSE_WORDS = 32 * 33;  // per epilogue warp: 32 rows x 32 words, padded row stride 33
 constexpr int XPOSE_BYTES = EPI_WARPS * XPOSE_WORDS * 4;
@@ -99,18 +101,18 @@ __device__ __forceinline__ void store_words_transposed(const uint32_t* xs, int l
 
 template <int EPI>
 __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t taddr, int mb, int nb, int quarter,
-                                              int lane, uint32_t* xs) {
+                                              int part, int lane, uint32_t* xs) {
   const int row0 = mb * BM + quarter * 32;  // first row of this warp
   const int row = row0 + lane;              // this thread's row (TMEM lane)
   if constexpr (EPI == EPI_STORE || EPI == EPI_QKV) {
     f16* out = reinterpret_cast<f16*>(p.out);
     const float rs = row_scale(p, row);
-#pragma unroll 1
-    for (int hh = 0; hh < BN / 128; ++hh) {
-      const int hc = nb * BN + hh * 128;  // first output column of this 128-column head
+    {
+      const int hh = part;                 // this warp's 128-column head of the tile
+      const int hc = nb * BN + hh * 128;  // first output column of this head
       const bool rope = (EPI == EPI_QKV) && hc < p.q_cols + p.k_cols;
       if (rope) {
-        // per-head RMSNorm (over the 128 columns, of the row-scaled values) then RoPE
+        // per-head RMSNorm of the row-scaled values: sum of squares in the row layout
         float ss = 0.f;
 #pragma unroll 1
         for (int c = 0; c < 128; c += 32) {
@@ -120,36 +122,69 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
 #pragma unroll
           for (int j = 0; j < 32; ++j) ss += __uint_as_float(v[j]) * __uint_as_float(v[j]);
         }
-        const float inv = rs * rsqrtf(ss * rs * rs * (1.f / 128.f) + p.eps);
-        const bf16* w = hc < p.q_cols ? p.q_norm : p.k_norm;
-        const int pos = row < p.M ? p.tok_pos[row] : 0;
-        const float2* cs = p.rope + static_cast<int64_t>(pos) * 64;
+        const float inv_row = rs * rsqrtf(ss * rs * rs * (1.f / 128.f) + p.eps);
+        const bf16* wgt = hc < p.q_cols ? p.q_norm : p.k_norm;
+        // the rotation runs in the transposed layout: lane L owns rows i*4 + L/8 and
+        // columns w4 .. w4+3 of each 32-column chunk, so RoPE-table reads and the
+        // stores are contiguous 8-lane row segments
+        const int w4 = (lane & 7) * 4;
+        float inv_i[8];
+        int pos_i[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int r = i * 4 + (lane >> 3);
+          inv_i[i] = __shfl_sync(0xffffffffu, inv_row, r);
+          pos_i[i] = row0 + r < p.M ? p.tok_pos[row0 + r] : 0;
+        }
 #pragma unroll 1
         for (int c = 0; c < 64; c += 32) {
-          uint32_t x1[32], x2[32];
-          tmem_ld32(taddr + hh * 128 + c, x1);
-          tmem_ld32(taddr + hh * 128 + 64 + c, x2);
-          tmem_ld_wait();
+          float4 x1[8], x2[8];
 #pragma unroll
-          for (int j = 0; j < 32; j += 2) {
-            float y1[2], y2[2];
+          for (int half = 0; half < 2; ++half) {
+            uint32_t v[32];
+            tmem_ld32(taddr + hh * 128 + half * 64 + c, v);
+            tmem_ld_wait();
 #pragma unroll
-            for (int e = 0; e < 2; ++e) {
-              const float a = __uint_as_float(x1[j + e]) * inv * __bfloat162float(w[c + j + e]);
-              const float b = __uint_as_float(x2[j + e]) * inv * __bfloat162float(w[64 + c + j + e]);
-              const float2 t = cs[c + j + e];
-              y1[e] = a * t.x - b * t.y;
-              y2[e] = b * t.x + a * t.y;
+            for (int j = 0; j < 32; ++j) xs[lane * 33 + j] = v[j];
+            __syncwarp();
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const int r = i * 4 + (lane >> 3);
+              const float4 t = make_float4(__uint_as_float(xs[r * 33 + w4]), __uint_as_float(xs[r * 33 + w4 + 1]),
+                                           __uint_as_float(xs[r * 33 + w4 + 2]), __uint_as_float(xs[r * 33 + w4 + 3]));
+              if (half == 0)
+                x1[i] = t;
+              else
+                x2[i] = t;
             }
-            xs[lane * 33 + j / 2] = pack_f16x2(y1[0], y1[1]);
-            xs[lane * 33 + 16 + j / 2] = pack_f16x2(y2[0], y2[1]);
+            __syncwarp();
           }
-          __syncwarp();
-          store_words_transposed(xs, lane, row0, p.M, [&](int r, int wd) {
-            const int col = hc + c + (wd < 16 ? 2 * wd : 64 + 2 * (wd - 16));
-            return out + static_cast<int64_t>(row0 + r) * p.ld_out + col;
-          });
-          __syncwarp();
+          float g1[4], g2[4];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            g1[k] = __bfloat162float(wgt[c + w4 + k]);
+            g2[k] = __bfloat162float(wgt[64 + c + w4 + k]);
+          }
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int r = i * 4 + (lane >> 3);
+            if (row0 + r < p.M) {
+              const float4* cs = reinterpret_cast<const float4*>(p.rope + static_cast<int64_t>(pos_i[i]) * 64 + c + w4);
+              const float4 c01 = cs[0], c23 = cs[1];  // (cos, sin) for frequencies c+w4 .. +3
+              const float cosv[4] = {c01.x, c01.z, c23.x, c23.z}, sinv[4] = {c01.y, c01.w, c23.y, c23.w};
+              const float a[4] = {x1[i].x, x1[i].y, x1[i].z, x1[i].w}, b[4] = {x2[i].x, x2[i].y, x2[i].z, x2[i].w};
+              float y1[4], y2[4];
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const float u = a[k] * inv_i[i] * g1[k], w = b[k] * inv_i[i] * g2[k];
+                y1[k] = u * cosv[k] - w * sinv[k];
+                y2[k] = w * cosv[k] + u * sinv[k];
+              }
+              f16* orow = out + static_cast<int64_t>(row0 + r) * p.ld_out + hc + c + w4;
+              *reinterpret_cast<uint2*>(orow) = make_uint2(pack_f16x2(y1[0], y1[1]), pack_f16x2(y1[2], y1[3]));
+              *reinterpret_cast<uint2*>(orow + 64) = make_uint2(pack_f16x2(y2[0], y2[1]), pack_f16x2(y2[2], y2[3]));
+            }
+          }
         }
       } else {
 #pragma unroll 1
@@ -187,16 +222,18 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
       return reinterpret_cast<float4*>(res + static_cast<int64_t>(row0 + i * 4 + (lane >> 3)) * p.ld_out + nb * BN +
                                        c + w4);
     };
+    const int cbeg = part * (BN / 2), cend = cbeg + BN / 2;  // this warp's half of the columns
     float4 cur[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i)
-      cur[i] = (row0 + i * 4 + (lane >> 3) < p.M) ? *rrow(i, 0) : make_float4(0.f, 0.f, 0.f, 0.f);
+      cur[i] = (row0 + i * 4 + (lane >> 3) < p.M) ? *rrow(i, cbeg) : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
+    for (int c = cbeg; c < cend; c += 32) {
       float4 nxt[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i)
-        nxt[i] = (c + 32 < BN && row0 + i * 4 + (lane >> 3) < p.M) ? *rrow(i, c + 32) : make_float4(0.f, 0.f, 0.f, 0.f);
+        nxt[i] = (c + 32 < cend && row0 + i * 4 + (lane >> 3) < p.M) ? *rrow(i, c + 32)
+                                                                      : make_float4(0.f, 0.f, 0.f, 0.f);
       uint32_t v[32];
       tmem_ld32(taddr + c, v);
       tmem_ld_wait();
@@ -242,14 +279,15 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
         t += __shfl_xor_sync(0xffffffffu, t, 2);
         t += __shfl_xor_sync(0xffffffffu, t, 4);
         const int r = i * 4 + (lane >> 3);
-        if ((lane & 7) == 0 && row0 + r < p.M) p.ss_out[static_cast<int64_t>(row0 + r) * p.ss_out_parts + nb] = t;
+        if ((lane & 7) == 0 && row0 + r < p.M)
+          p.ss_out[static_cast<int64_t>(row0 + r) * p.ss_out_parts + nb * GEMM_SS_PER_TILE + part] = t;
       }
     }
   } else {  // EPI_SWIGLU: columns 0..127 gate, 128..255 up of the same 128 outputs
     f16* out = reinterpret_cast<f16*>(p.out);
     const float rs = row_scale(p, row);
-#pragma unroll 1
-    for (int c = 0; c < BN / 2; c += 64) {
+    {
+      const int c = part * 64;  // this warp's 64 of the tile's 128 outputs
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         uint32_t g[32], u[32];
@@ -388,8 +426,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_wait(drain_bar, 0, p.err, ok ? p.timeout_ns : 100000000ull);
     }
   } else {
-    // ---------------- epilogue warps 2..5 -> TMEM lane quarters 2,3,0,1
+    // ---------------- epilogue warps 2..9 -> TMEM lane quarters 2,3,0,1 (x2), column halves 0/1
     const int quarter = warp & 3;
+    const int part = (warp - 2) >> 2;
     uint32_t* xs = xpose + (warp - 2) * XPOSE_WORDS;
     int local = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x, ++local) {
@@ -400,7 +439,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (!mbar_wait(tfull_bar(acc), acc_phase, p.err, p.timeout_ns)) break;
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
-      epilogue_tile<EPI>(p, taddr, mb, nb, quarter, lane, xs);
+      epilogue_tile<EPI>(p, taddr, mb, nb, quarter, part, lane, xs);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty_bar(acc));
