@@ -130,8 +130,9 @@ void free_workspace(Workspace& w) {
   dev_free(w.q_off); dev_free(w.q_tok); dev_free(w.doc_ids); dev_free(w.scores);
   dev_free(w.pair_slot); dev_free(w.perm); dev_free(w.sorted_slot); dev_free(w.tok_off);
   dev_free(w.tok_id); dev_free(w.tok_pos); dev_free(w.tok_pair); dev_free(w.doc_count);
-  dev_free(w.items); dev_free(w.err);
+  dev_free(w.items); dev_free(w.tiles); dev_free(w.err);
   host_free(w.h_tok_off); host_free(w.h_sorted_slot); host_free(w.h_err); host_free(w.h_items);
+  host_free(w.h_tiles);
   w = Workspace{};
 }
 
@@ -146,6 +147,7 @@ void free_model(Model* m) {
 
 void free_store(Store* s) {
   dev_free(s->pool); dev_free(s->d_slot_of); dev_free(s->d_slot_m); dev_free(s->d_slot_row); dev_free(s->d_slot_ok);
+  dev_free(s->d_range);
 }
 
 dopr_status build_weight_maps(Model* m) {
@@ -205,18 +207,18 @@ dopr_status ensure_call_buffers(Model* m, int64_t n_pairs, int64_t n_tokens, int
     STATUS_TRY(dev_alloc(&w.perm, cap));
     STATUS_TRY(dev_alloc(&w.sorted_slot, cap));
     STATUS_TRY(dev_alloc(&w.tok_off, cap + 1));
-    STATUS_TRY(dev_alloc(&w.items, cap + 1024));
+    STATUS_TRY(dev_alloc(&w.items, 2 * (cap + 1024)));
     w.pair_cap = cap;
-    w.item_cap = cap + 1024;
+    w.item_cap = 2 * (cap + 1024);
   }
   if (n_pairs > w.h_pair_cap) {
     const int64_t cap = std::max<int64_t>(n_pairs, 2 * w.h_pair_cap);
     host_free(w.h_tok_off); host_free(w.h_sorted_slot); host_free(w.h_items);
     STATUS_TRY(host_alloc(&w.h_tok_off, cap + 1));
     STATUS_TRY(host_alloc(&w.h_sorted_slot, cap));
-    STATUS_TRY(host_alloc(&w.h_items, cap + 1024));
+    STATUS_TRY(host_alloc(&w.h_items, 2 * (cap + 1024)));
     w.h_pair_cap = cap;
-    w.h_item_cap = cap + 1024;
+    w.h_item_cap = 2 * (cap + 1024);
   }
   if (n_tokens > w.tok_cap) {
     const int64_t cap = std::max<int64_t>(n_tokens, 2 * w.tok_cap);
@@ -225,6 +227,14 @@ dopr_status ensure_call_buffers(Model* m, int64_t n_pairs, int64_t n_tokens, int
     STATUS_TRY(dev_alloc(&w.tok_pos, cap));
     STATUS_TRY(dev_alloc(&w.tok_pair, cap));
     w.tok_cap = cap;
+  }
+  if (n_tokens > w.tile_cap) {  // a tile holds at least one token
+    const int64_t cap = std::max<int64_t>(n_tokens, 2 * w.tile_cap);
+    dev_free(w.tiles);
+    host_free(w.h_tiles);
+    STATUS_TRY(dev_alloc(&w.tiles, cap));
+    STATUS_TRY(host_alloc(&w.h_tiles, cap));
+    w.tile_cap = cap;
   }
   if (n_qtokens > w.qtok_cap) {
     const int64_t cap = std::max<int64_t>(n_qtokens, 2 * w.qtok_cap);
@@ -347,10 +357,54 @@ PackArgs pack_args(Model* m, Store* s, int32_t n, const int32_t* dqo, const int3
 
 struct Plan {
   int64_t n_tokens = 0;
-  std::vector<int32_t> chunk_pair;  // chunk c covers sorted pairs [chunk_pair[c], chunk_pair[c+1])
-  std::vector<int32_t> chunk_item;  // and attention items [chunk_item[c], chunk_item[c+1])
-  int32_t n_items = 0;
+  std::vector<int32_t> chunk_pair;   // chunk c covers sorted pairs [chunk_pair[c], chunk_pair[c+1])
+  std::vector<int32_t> chunk_item;   // and attention items [chunk_item[c], chunk_item[c+1]) (every pair)
+  std::vector<int32_t> chunk_litem;  // mma.sync-kernel items [chunk_litem[c], chunk_litem[c+1])
+  std::vector<int32_t> chunk_tile;   // tensor-core tiles [chunk_tile[c], chunk_tile[c+1])
+  int32_t n_items = 0, n_litems = 0, n_tiles = 0;
 };
+
+// Cut the sorted pairs [pb, pe) of one document (chunk-relative token offsets
+// from `to`, t0 the chunk's first token) into tensor-core tiles of at most TT
+// tokens and ATTN_TC_MAX_KEYS key columns, and runs of pairs that do not fit
+// the key budget into mma.sync-kernel items.
+void plan_attention(const int32_t* to, int32_t t0, int32_t pb, int32_t pe, int32_t slot, int32_t m, int TT,
+                    std::vector<AttnTile>& tiles, std::vector<AttnItem>& litems) {
+  auto c16 = [](int x) { return (x + 15) & ~15; };
+  auto fits = [&](int32_t p) { return TT > 0 && attn_tc_pair_fits(m, to[p + 1] - to[p]); };
+  const int pre64 = ((m + 63) / 64) * 64;
+  int32_t p = pb;
+  while (p < pe) {
+    int32_t q = p + 1;
+    if (!fits(p)) {
+      while (q < pe && q - p < ATTN_MAX_PAIRS && !fits(q)) ++q;
+      litems.push_back(AttnItem{p, q, slot, m});
+      p = q;
+      continue;
+    }
+    while (q < pe && fits(q)) ++q;
+    const int32_t end = to[q] - t0;
+    int32_t tok = to[p] - t0, pf = p;
+    while (tok < end) {
+      while (to[pf + 1] - t0 <= tok) ++pf;
+      int32_t n = 0, closed = 0, keys = 0, pp = pf;
+      while (n < TT && tok + n < end) {
+        const int32_t t = tok + n;
+        while (to[pp + 1] - t0 <= t) {  // pair pp lies wholly in the tile: its full segment
+          closed += c16(to[pp + 1] - to[pp]);
+          ++pp;
+        }
+        const int32_t k = pre64 + closed + c16(t - (to[pp] - t0) + 1);
+        if (k > ATTN_TC_MAX_KEYS) break;
+        keys = k;
+        ++n;
+      }
+      tiles.push_back(AttnTile{tok, n, pf, slot, m, keys});
+      tok += n;
+    }
+    p = q;
+  }
+}
 
 // Steps 1-4 of the engine.  Inputs are device pointers.  On return the packed
 // plan is on the device and the chunking in `plan`.
@@ -370,10 +424,16 @@ dopr_status run_packer(Model* m, Store* s, int32_t n, const int32_t* dqo, const 
   STATUS_TRY(ensure_call_buffers(m, n, plan.n_tokens, 0, 0));
   a = pack_args(m, s, n, dqo, dqt, ddoc);
   CUDA_TRY(prof_launch(m, K_PACK, 1, 0.0, 16.0 * plan.n_tokens, st, [&] { return launch_pack_tokens(a, st); }));
-  // chunks of whole pairs, then attention items (runs of one doc, <= ATTN_MAX_PAIRS)
+  // chunks of whole pairs, then attention items (runs of one doc, <= ATTN_MAX_PAIRS),
+  // and per chunk the tensor-core tiles and the mma.sync kernel's items
   const int cap = w.chunk_cap;
+  const int TT = attn_tc_rows_per_head(m->cfg.n_q_heads / m->cfg.n_kv_heads);
   plan.chunk_pair.assign(1, 0);
   plan.chunk_item.assign(1, 0);
+  plan.chunk_litem.assign(1, 0);
+  plan.chunk_tile.assign(1, 0);
+  std::vector<AttnTile> tiles;
+  std::vector<AttnItem> litems;
   int32_t items = 0;
   int32_t s0 = 0;
   while (s0 < n) {
@@ -384,21 +444,31 @@ dopr_status run_packer(Model* m, Store* s, int32_t n, const int32_t* dqo, const 
     int32_t i = s0;
     while (i < s1) {
       int32_t j = i + 1;
-      while (j < s1 && j - i < ATTN_MAX_PAIRS && w.h_sorted_slot[j] == w.h_sorted_slot[i]) ++j;
-      AttnItem it;
-      it.pair_begin = i;
-      it.pair_end = j;
-      it.slot = w.h_sorted_slot[i];
-      it.m = s->slot_m[it.slot];
-      w.h_items[items++] = it;
+      while (j < s1 && w.h_sorted_slot[j] == w.h_sorted_slot[i]) ++j;  // the document's run in this chunk
+      const int32_t slot = w.h_sorted_slot[i], mm = s->slot_m[slot];
+      for (int32_t a = i; a < j; a += ATTN_MAX_PAIRS)
+        w.h_items[items++] = AttnItem{a, std::min(j, a + ATTN_MAX_PAIRS), slot, mm};
+      plan_attention(w.h_tok_off, w.h_tok_off[s0], i, j, slot, mm, TT, tiles, litems);
       i = j;
     }
     plan.chunk_pair.push_back(s1);
     plan.chunk_item.push_back(items);
+    plan.chunk_litem.push_back((int32_t)litems.size());
+    plan.chunk_tile.push_back((int32_t)tiles.size());
     s0 = s1;
   }
   plan.n_items = items;
-  if (items > 0) CUDA_TRY(cudaMemcpyAsync(w.items, w.h_items, sizeof(AttnItem) * items, cudaMemcpyHostToDevice, st));
+  plan.n_litems = (int32_t)litems.size();
+  plan.n_tiles = (int32_t)tiles.size();
+  if (items + plan.n_litems > w.item_cap || items + plan.n_litems > w.h_item_cap || plan.n_tiles > w.tile_cap)
+    return fail(DOPR_ERR_UNSUPPORTED, "attention plan exceeds its buffers");
+  std::copy(litems.begin(), litems.end(), w.h_items + items);
+  std::copy(tiles.begin(), tiles.end(), w.h_tiles);
+  if (items + plan.n_litems > 0)
+    CUDA_TRY(cudaMemcpyAsync(w.items, w.h_items, sizeof(AttnItem) * (items + plan.n_litems), cudaMemcpyHostToDevice,
+                             st));
+  if (plan.n_tiles > 0)
+    CUDA_TRY(cudaMemcpyAsync(w.tiles, w.h_tiles, sizeof(AttnTile) * plan.n_tiles, cudaMemcpyHostToDevice, st));
   return DOPR_OK;
 }
 
@@ -445,6 +515,28 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     const double attn_flops_last = 4.0 * HEAD_DIM * Hq * last_keys;
     const double attn_bytes_last = np * 2.0 * Hq * HEAD_DIM * 2 + T * 2.0 * Hkv * HEAD_DIM * 2 +
                                    prefix_rows * Hkv * 2 * HEAD_DIM * 2;
+    // this chunk's packed QKV buffer as TMA maps for the tensor-core attention:
+    // Q boxes of 128 / G rows per q head, own-key boxes of 16 rows
+    const int TT = attn_tc_rows_per_head(Hq / Hkv);
+    CUtensorMap tm_q{}, tm_kv{};
+    const int n_tiles = plan.chunk_tile[ci + 1] - plan.chunk_tile[ci];
+    if (n_tiles > 0 &&
+        !(make_tmap_16b_2d(&tm_q, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, TT, true, true) &&
+          make_tmap_16b_2d(&tm_kv, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, 16, true, true)))
+      return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for the QKV buffer");
+    AttnTcArgs ta{};
+    ta.tiles = w.tiles + plan.chunk_tile[ci];
+    ta.n_units = n_tiles * Hkv;
+    ta.tok_off = w.tok_off;
+    ta.tok0 = t0;
+    ta.out = w.o;
+    ta.ld_out = m->o_dim;
+    ta.slot_row = s->d_slot_row;
+    ta.Hq = Hq;
+    ta.Hkv = Hkv;
+    ta.err = w.err;
+    const int32_t li0 = plan.n_items + plan.chunk_litem[ci];
+    const int32_t n_litems = plan.chunk_litem[ci + 1] - plan.chunk_litem[ci];
     const auto op_last = gemm_cost(np, H, m->o_dim, np * H * 10.0);
     const auto gu_last = gemm_cost(np, 2.0 * F, H, np * F * 2.0);
     const auto dn_last = gemm_cost(np, H, F, np * H * 8.0);
@@ -473,8 +565,8 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       CUDA_TRY(prof_launch(m, K_GEMM_QKV, 1, qkv.first, qkv.second, st,
                            [&] { return launch_gemm(EPI_QKV, w.tm_xn, m->tm_qkv[l], pq, sms, st); }));
       AttnArgs aa{};
-      aa.items = w.items + plan.chunk_item[ci];
-      aa.n_items = plan.chunk_item[ci + 1] - plan.chunk_item[ci];
+      aa.items = w.items + (last ? plan.chunk_item[ci] : li0);
+      aa.n_items = last ? plan.chunk_item[ci + 1] - plan.chunk_item[ci] : n_litems;
       aa.tok_off = w.tok_off;
       aa.tok0 = t0;
       aa.qkv = w.qkv;
@@ -490,9 +582,20 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       aa.score_only = last ? 1 : 0;
       aa.pair_base = s0;
       aa.err = w.err;
-      CUDA_TRY(prof_launch(m, K_ATTENTION, 1, last ? attn_flops_last : attn_flops,
+      const int attn_launches = (!last && ta.n_units > 0 ? 1 : 0) + (aa.n_items > 0 ? 1 : 0);
+      CUDA_TRY(prof_launch(m, K_ATTENTION, attn_launches, last ? attn_flops_last : attn_flops,
                            last ? attn_bytes_last : attn_bytes, st,
-                           [&] { return launch_attention(s->tm_pool, aa, st); }));
+                           [&] {
+                             // every layer but the last: tensor-core tiles, then the pairs beyond
+                             // their key budget; the last layer: score-token rows of every pair
+                             cudaError_t e = cudaSuccess;
+                             if (!last && ta.n_units > 0) {
+                               ta.layer = l;
+                               e = launch_attention_tc(tm_q, tm_kv, s->tm_pool, ta, sms, st);
+                             }
+                             if (e == cudaSuccess && aa.n_items > 0) e = launch_attention(s->tm_pool, aa, st);
+                             return e;
+                           }));
       const float* ss_pre = l == 0 ? w.ss_e : w.ss_a;  // the attention norm of this layer
       const int ss_pre_parts = l == 0 ? 1 : parts;
       float* resid = w.r;
@@ -620,7 +723,7 @@ dopr_status dopr_model_create(const dopr_model_config* cfg, dopr_model** out) {
   };
   cudaGetDevice(&m->device);
   cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
-  guard(gemm_setup() == cudaSuccess && attn_setup() == cudaSuccess
+  guard(gemm_setup() == cudaSuccess && attn_setup() == cudaSuccess && attn_tc_setup() == cudaSuccess
             ? DOPR_OK
             : fail(DOPR_ERR_CUDA, "kernel attribute setup failed: %s", cudaGetErrorString(cudaGetLastError())));
   if (st == DOPR_OK &&
@@ -750,7 +853,7 @@ dopr_status dopr_store_create(const dopr_model_config* cfg, int64_t max_doc_id, 
   };
   if (guard(dev_alloc(&s->pool, (size_t)std::max<int64_t>(s->pool_bytes, 256))) &&
       guard(dev_alloc(&s->d_slot_of, nd)) && guard(dev_alloc(&s->d_slot_m, nd)) &&
-      guard(dev_alloc(&s->d_slot_row, nd)) && guard(dev_alloc(&s->d_slot_ok, nd))) {
+      guard(dev_alloc(&s->d_slot_row, nd)) && guard(dev_alloc(&s->d_slot_ok, nd)) && guard(dev_alloc(&s->d_range, 1))) {
     if (cudaMemset(s->d_slot_of, 0xFF, nd * sizeof(int32_t)) != cudaSuccess ||
         cudaMemset(s->d_slot_ok, 0, nd) != cudaSuccess || cudaMemset(s->d_slot_m, 0, nd * sizeof(int32_t)) ||
         cudaMemset(s->pool, 0, (size_t)std::max<int64_t>(s->pool_bytes, 256)) != cudaSuccess)
@@ -758,7 +861,7 @@ dopr_status dopr_store_create(const dopr_model_config* cfg, int64_t max_doc_id, 
   }
   if (st == DOPR_OK &&
       !make_tmap_16b_2d(&s->tm_pool, s->pool, HEAD_DIM, std::max<int64_t>(s->pool_rows, 1), HEAD_DIM * 2, 64, 64, true,
-                        false))
+                        true))
     guard(fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for the store pool"));
   if (st != DOPR_OK) {
     free_store(s);
@@ -806,7 +909,7 @@ dopr_status dopr_store_put(dopr_store* s, int64_t doc_id, int32_t m, int32_t lay
   }
   if (m > 0) {
     const size_t bytes = (size_t)m * Hkv * HEAD_DIM * 2;
-    bf16* base = reinterpret_cast<bf16*>(s->pool) + (size_t)(s->slot_row[slot] + layer * rows_per_layer) * HEAD_DIM;
+    f16* base = reinterpret_cast<f16*>(s->pool) + (size_t)(s->slot_row[slot] + layer * rows_per_layer) * HEAD_DIM;
     const bf16 *dk = static_cast<const bf16*>(k), *dv = static_cast<const bf16*>(v);
     bf16* stage = nullptr;
     if (!src_on_device) {
@@ -820,10 +923,24 @@ dopr_status dopr_store_put(dopr_store* s, int64_t doc_id, int32_t m, int32_t lay
       dk = stage;
       dv = stage + bytes / 2;
     }
-    cudaError_t e = launch_store_transpose(dk, dv, m, (int)Hkv, base, base + (size_t)Hkv * m * HEAD_DIM, 0);
-    if (e == cudaSuccess) e = cudaStreamSynchronize(0);
+    int range = 0;
+    cudaError_t e = cudaMemsetAsync(s->d_range, 0, sizeof(int), 0);
+    if (e == cudaSuccess)
+      e = launch_store_transpose(dk, dv, m, (int)Hkv, base, base + (size_t)Hkv * m * HEAD_DIM, s->d_range, 0);
+    if (e == cudaSuccess) e = cudaMemcpy(&range, s->d_range, sizeof(int), cudaMemcpyDeviceToHost);
     if (stage) cudaFree(stage);
     if (e != cudaSuccess) return fail(DOPR_ERR_CUDA, "prefix store copy failed: %s", cudaGetErrorString(e));
+    if (range) {
+      // the layer now holds clamped data: mark it missing until a valid put replaces it
+      if (s->slot_layers[slot][layer] && s->slot_ok[slot]) {
+        s->slot_ok[slot] = 0;
+        const uint8_t zero = 0;
+        CUDA_TRY(cudaMemcpy(s->d_slot_ok + slot, &zero, 1, cudaMemcpyHostToDevice));
+      }
+      s->slot_layers[slot][layer] = 0;
+      return fail(DOPR_ERR_INVALID_ARG, "doc %lld layer %d: a prefix value is not finite or exceeds the fp16 range",
+                  (long long)doc_id, layer);
+    }
   }
   if (!s->slot_layers[slot][layer]) {
     s->slot_layers[slot][layer] = 1;

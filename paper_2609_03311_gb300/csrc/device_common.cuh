@@ -156,6 +156,20 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr) {
   return d;
 }
 
+// Shared-memory matrix descriptor: MN-major operand (the N index contiguous),
+// 128-byte swizzle.  An atom is 8 rows along K of 64 16-bit N-elements (128 B);
+// `lbo` is the byte stride between 64-element groups along N, `sbo` the byte
+// stride between 8-row groups along K.
+__device__ __forceinline__ uint64_t umma_desc_sw128_mn(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(2) << 61;
+  return d;
+}
+
 // Instruction descriptor, kind::f16: D fp32, A and B fp16 (format code 0), both K-major.
 __host__ __device__ constexpr uint32_t umma_idesc_f16(int M, int N) {
   return (1u << 4)                                  // D format: f32
@@ -164,6 +178,9 @@ __host__ __device__ constexpr uint32_t umma_idesc_f16(int M, int N) {
          | (static_cast<uint32_t>(N >> 3) << 17)    // N / 8
          | (static_cast<uint32_t>(M >> 4) << 24);   // M / 16
 }
+
+// As umma_idesc_f16 with B MN-major (the "transpose B" bit).
+__host__ __device__ constexpr uint32_t umma_idesc_f16_bmn(int M, int N) { return umma_idesc_f16(M, N) | (1u << 16); }
 
 // 32 lanes x 32 columns of 32-bit TMEM data starting at taddr; thread i of the
 // warp receives lane (taddr.lane + i), columns taddr.col .. +31.

@@ -29,12 +29,28 @@ struct AttnItem {
   int32_t m;                     // its prefix length
 };
 
+// Tensor-core attention (k_attn_tc.cu).  A tile is up to 128 / G consecutive
+// packed tokens of pairs of one document; its keys are the prefix (ceil64(m)
+// columns) then one segment per pair it touches, from the pair's first token to
+// the tile's last, each padded to a multiple of 16 columns.  Pairs whose own
+// segment can exceed the key budget take the mma.sync kernel (k_attn.cu).
+constexpr int ATTN_TC_MAX_KEYS = 256;
+struct AttnTile {
+  int32_t tok_begin;   // first token, relative to the chunk
+  int32_t n_tok;       // tokens in the tile (<= 128 / G)
+  int32_t pair_first;  // sorted index of the pair holding tok_begin
+  int32_t slot;        // store slot of the document
+  int32_t m;           // its prefix length
+  int32_t n_keys;      // key columns (multiple of 16, <= ATTN_TC_MAX_KEYS)
+};
+
 struct Store {
   dopr_model_config cfg{};
   int device = 0;
   int64_t max_doc_id = 0;
-  int64_t pool_bytes = 0, pool_rows = 0, used_rows = 0;  // rows of 128 bf16 (256 B)
-  uint8_t* pool = nullptr;
+  int64_t pool_bytes = 0, pool_rows = 0, used_rows = 0;  // rows of 128 fp16 (256 B)
+  uint8_t* pool = nullptr;          // prefix K/V as fp16 (converted from the bf16 the caller passes)
+  int* d_range = nullptr;           // set by the put conversion when a value leaves the fp16 range
   int32_t* d_slot_of = nullptr;     // [max_doc_id+1] doc -> slot, -1 absent
   int32_t* d_slot_m = nullptr;      // [max_doc_id+1] per slot prefix length
   int64_t* d_slot_row = nullptr;    // [max_doc_id+1] first pool row of the slot block
@@ -77,13 +93,16 @@ struct Workspace {
   int32_t* tok_pos = nullptr;
   int32_t* tok_pair = nullptr;
   int32_t* doc_count = nullptr;  // [max_doc_id+1] counting-sort buckets
-  AttnItem* items = nullptr;
+  AttnItem* items = nullptr;     // all items of the call, then the mma.sync kernel's items
+  AttnTile* tiles = nullptr;     // tensor-core attention tiles of the call
+  int64_t tile_cap = 0;
   int* err = nullptr;
   // pinned host staging
   int32_t* h_tok_off = nullptr;
   int32_t* h_sorted_slot = nullptr;
   int* h_err = nullptr;
   AttnItem* h_items = nullptr;
+  AttnTile* h_tiles = nullptr;
   int64_t h_pair_cap = 0, h_item_cap = 0;
 };
 
@@ -187,7 +206,9 @@ cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0
 // dst_ss[i] = ss[row(i)] (parts floats), row(i) = tok_off[p_begin+i+1]-1-tok0.
 cudaError_t launch_gather_score_rows(const float* r, const float* ss, int H, int parts, const int32_t* tok_off,
                                      int tok0, int p_begin, int p_end, float* dst_r, float* dst_ss, cudaStream_t st);
-cudaError_t launch_store_transpose(const bf16* k, const bf16* v, int m, int Hkv, bf16* dk, bf16* dv,
+// [m][Hkv][128] bf16 -> [Hkv][m][128] fp16 for K and V; *range |= 1 when a value
+// is not finite or exceeds the fp16 range (|x| > 65504).
+cudaError_t launch_store_transpose(const bf16* k, const bf16* v, int m, int Hkv, f16* dk, f16* dv, int* range,
                                    cudaStream_t st);
 
 // Attention.
@@ -209,6 +230,30 @@ struct AttnArgs {
 };
 cudaError_t attn_setup();
 cudaError_t launch_attention(const CUtensorMap& tm_pool, const AttnArgs& a, cudaStream_t st);
+
+// Arguments of the tensor-core attention kernel.
+struct AttnTcArgs {
+  const AttnTile* tiles;
+  int n_units;             // tiles x kv heads
+  const int32_t* tok_off;  // sorted pair -> first packed token
+  int32_t tok0;            // first packed token of this chunk
+  f16* out;
+  int ld_out;
+  const int64_t* slot_row;
+  int layer, Hq, Hkv;
+  int* err;
+};
+// Q rows per head in a 128-row tile; 0 when the group size does not divide 128 into boxes of >= 8 rows.
+inline int attn_tc_rows_per_head(int G) { return (G >= 1 && G <= 16 && 128 % G == 0) ? 128 / G : 0; }
+// Whether a pair of T tokens (query + score token) on a prefix of m keys fits one tile's key budget.
+inline bool attn_tc_pair_fits(int m, int T) {
+  return ((m + 63) / 64) * 64 + ((T + 15) / 16) * 16 <= ATTN_TC_MAX_KEYS;
+}
+cudaError_t attn_tc_setup();
+// tm_q: the chunk's packed QKV buffer, box 64 columns x (128 / G) rows; tm_kv: the same
+// buffer, box 64 x 16; tm_pool: the store pool, box 64 x 64 (all fp16, 128-byte swizzle).
+cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool,
+                                const AttnTcArgs& a, int num_sms, cudaStream_t st);
 
 // Packer.
 struct PackArgs {

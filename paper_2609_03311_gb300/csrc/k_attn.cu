@@ -17,9 +17,10 @@
 // 32-key blocks, then its own causal keys in 16-key blocks, with the online
 // (running max / running sum) softmax.  Pairs longer
 // than OWN_CAP stream their own keys in OWN_CAP chunks per 64-row group.
-// Scores and P.V use warp-level fp16 mma with fp32 accumulation (the stored
-// bf16 prefix is widened to fp16 in shared memory after it lands); row maxima
-// and sums use quad shuffles.
+// Scores and P.V use warp-level fp16 mma with fp32 accumulation (the store
+// keeps the prefix as fp16); row maxima and sums use quad shuffles.  This
+// kernel takes the pairs whose keys exceed the tensor-core kernel's budget and
+// the score-token rows of the last layer.
 #include <math.h>
 
 #include "device_common.cuh"
@@ -252,25 +253,14 @@ __global__ void __launch_bounds__(THREADS, DOPR_ATTN_MIN_BLOCKS) k_attn(const __
       if (tid == 0) mbar_wait(bar, 0, a.err, 100000000ull);  // let the copies land first
       return;
     }
-    // The stored prefix is bf16: widen it to fp16 in place (element-wise, so the
-    // swizzled layout is unchanged).  Rows m .. nbox*64-1 of the boxes hold other
-    // data: zero them so masked keys contribute exactly 0 to P.V.
+    // Rows m .. nbox*64-1 of the boxes hold other data: zero them so masked keys
+    // contribute exactly 0 to P.V.
     uint8_t* gk = smem;
     uint8_t* gv = smem + a.mpad_cap * ROW_BYTES;
-    for (int i = tid; i < nbox * 64 * 16; i += THREADS) {
+    for (int i = m * 16 + tid; i < nbox * 64 * 16; i += THREADS) {
       const int r = i / 16, c = i % 16;
-      uint4* pk = reinterpret_cast<uint4*>(gk + off_pre(r, c));
-      uint4* pv = reinterpret_cast<uint4*>(gv + off_pre(r, c));
-      if (r >= m) {
-        *pk = make_uint4(0, 0, 0, 0);
-        *pv = make_uint4(0, 0, 0, 0);
-      } else {
-        uint4 x = *pk, y = *pv;
-        x = make_uint4(bf16x2_to_f16x2(x.x), bf16x2_to_f16x2(x.y), bf16x2_to_f16x2(x.z), bf16x2_to_f16x2(x.w));
-        y = make_uint4(bf16x2_to_f16x2(y.x), bf16x2_to_f16x2(y.y), bf16x2_to_f16x2(y.z), bf16x2_to_f16x2(y.w));
-        *pk = x;
-        *pv = y;
-      }
+      *reinterpret_cast<uint4*>(gk + off_pre(r, c)) = make_uint4(0, 0, 0, 0);
+      *reinterpret_cast<uint4*>(gv + off_pre(r, c)) = make_uint4(0, 0, 0, 0);
     }
     // (the barrier before the first own-key load orders these writes)
   }

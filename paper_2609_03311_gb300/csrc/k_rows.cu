@@ -109,10 +109,23 @@ __global__ void __launch_bounds__(ROW_WARPS * 32)
   for (int c = lane; c < parts; c += 32) dst_ss[static_cast<int64_t>(i) * parts + c] = ss[row * parts + c];
 }
 
-// [m][Hkv][128] -> [Hkv][m][128] for K and V (16-byte granules).
+// [m][Hkv][128] bf16 -> [Hkv][m][128] fp16 for K and V (8 elements per thread).
+// bf16 -> fp16 is exact for every value of fp16's normal range; values beyond it
+// (or not finite) are flagged in *range.
+__device__ __forceinline__ uint4 bf16x8_to_f16x8(uint4 x, int& bad) {
+  uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[i]));
+    bad |= !(fabsf(f.x) <= 65504.f) || !(fabsf(f.y) <= 65504.f);
+    w[i] = pack_f16x2(f.x, f.y);
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
 __global__ void k_store_transpose(const uint4* __restrict__ k, const uint4* __restrict__ v, int m, int Hkv,
-                                  uint4* __restrict__ dk, uint4* __restrict__ dv) {
+                                  uint4* __restrict__ dk, uint4* __restrict__ dv, int* range) {
   const int64_t n = static_cast<int64_t>(m) * Hkv * (HEAD_DIM / 8);
+  int bad = 0;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const int c = static_cast<int>(i % (HEAD_DIM / 8));
@@ -120,9 +133,10 @@ __global__ void k_store_transpose(const uint4* __restrict__ k, const uint4* __re
     const int h = static_cast<int>(rest % Hkv);
     const int64_t j = rest / Hkv;
     const int64_t o = (static_cast<int64_t>(h) * m + j) * (HEAD_DIM / 8) + c;
-    dk[o] = k[i];
-    dv[o] = v[i];
+    dk[o] = bf16x8_to_f16x8(k[i], bad);
+    dv[o] = bf16x8_to_f16x8(v[i], bad);
   }
+  if (bad) atomicOr(range, 1);
 }
 
 // Test kernel: one bounded wait on an mbarrier that is never completed.
@@ -174,13 +188,13 @@ cudaError_t launch_gather_score_rows(const float* r, const float* ss, int H, int
   return cudaGetLastError();
 }
 
-cudaError_t launch_store_transpose(const bf16* k, const bf16* v, int m, int Hkv, bf16* dk, bf16* dv,
+cudaError_t launch_store_transpose(const bf16* k, const bf16* v, int m, int Hkv, f16* dk, f16* dv, int* range,
                                    cudaStream_t st) {
   if (m <= 0) return cudaSuccess;
   const int64_t n = static_cast<int64_t>(m) * Hkv * (HEAD_DIM / 8);
   const int blocks = static_cast<int>((n + 255) / 256);
   k_store_transpose<<<blocks, 256, 0, st>>>(reinterpret_cast<const uint4*>(k), reinterpret_cast<const uint4*>(v), m,
-                                            Hkv, reinterpret_cast<uint4*>(dk), reinterpret_cast<uint4*>(dv));
+                                            Hkv, reinterpret_cast<uint4*>(dk), reinterpret_cast<uint4*>(dv), range);
   return cudaGetLastError();
 }
 
