@@ -368,8 +368,8 @@ struct Plan {
 // from `to`, t0 the chunk's first token) into tensor-core tiles of at most TT
 // tokens and ATTN_TC_MAX_KEYS key columns, and runs of pairs that do not fit
 // the key budget into mma.sync-kernel items.
-void plan_attention(const int32_t* to, int32_t t0, int32_t pb, int32_t pe, int32_t slot, int32_t m, int TT,
-                    std::vector<AttnTile>& tiles, std::vector<AttnItem>& litems) {
+void plan_attention(const int32_t* to, int32_t t0, int32_t pb, int32_t pe, int32_t slot, int32_t m, int64_t pool_base,
+                    int TT, std::vector<AttnTile>& tiles, std::vector<AttnItem>& litems) {
   auto c16 = [](int x) { return (x + 15) & ~15; };
   auto fits = [&](int32_t p) { return TT > 0 && attn_tc_pair_fits(m, to[p + 1] - to[p]); };
   const int pre64 = ((m + 63) / 64) * 64;
@@ -399,7 +399,17 @@ void plan_attention(const int32_t* to, int32_t t0, int32_t pb, int32_t pe, int32
         keys = k;
         ++n;
       }
-      tiles.push_back(AttnTile{tok, n, pf, slot, m, keys});
+      AttnTile tl{};
+      tl.pool_base = pool_base;
+      tl.tok_begin = tok;
+      tl.n_tok = n;
+      tl.m = m;
+      tl.n_keys = keys;
+      for (int32_t sp = pf; to[sp] - t0 < tok + n; ++sp) {
+        const int32_t ps = to[sp] - t0, nvis = std::min(to[sp + 1] - t0, tok + n) - ps;
+        tl.seg[tl.n_seg++] = (int32_t)(((uint32_t)nvis << 16) | (uint16_t)(int16_t)(ps - tok));
+      }
+      tiles.push_back(tl);
       tok += n;
     }
     p = q;
@@ -448,7 +458,7 @@ dopr_status run_packer(Model* m, Store* s, int32_t n, const int32_t* dqo, const 
       const int32_t slot = w.h_sorted_slot[i], mm = s->slot_m[slot];
       for (int32_t a = i; a < j; a += ATTN_MAX_PAIRS)
         w.h_items[items++] = AttnItem{a, std::min(j, a + ATTN_MAX_PAIRS), slot, mm};
-      plan_attention(w.h_tok_off, w.h_tok_off[s0], i, j, slot, mm, TT, tiles, litems);
+      plan_attention(w.h_tok_off, w.h_tok_off[s0], i, j, slot, mm, s->slot_row[slot], TT, tiles, litems);
       i = j;
     }
     plan.chunk_pair.push_back(s1);
@@ -527,11 +537,8 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     AttnTcArgs ta{};
     ta.tiles = w.tiles + plan.chunk_tile[ci];
     ta.n_units = n_tiles * Hkv;
-    ta.tok_off = w.tok_off;
-    ta.tok0 = t0;
     ta.out = w.o;
     ta.ld_out = m->o_dim;
-    ta.slot_row = s->d_slot_row;
     ta.Hq = Hq;
     ta.Hkv = Hkv;
     ta.err = w.err;

@@ -35,13 +35,18 @@ struct AttnItem {
 // the tile's last, each padded to a multiple of 16 columns.  Pairs whose own
 // segment can exceed the key budget take the mma.sync kernel (k_attn.cu).
 constexpr int ATTN_TC_MAX_KEYS = 256;
-struct AttnTile {
+constexpr int ATTN_TC_MAX_SEGS = 16;  // own segments are >= 16 columns each
+struct __align__(16) AttnTile {
+  int64_t pool_base;   // first store-pool row of the document's slot
   int32_t tok_begin;   // first token, relative to the chunk
   int32_t n_tok;       // tokens in the tile (<= 128 / G)
-  int32_t pair_first;  // sorted index of the pair holding tok_begin
-  int32_t slot;        // store slot of the document
-  int32_t m;           // its prefix length
+  int32_t m;           // the document's prefix length
   int32_t n_keys;      // key columns (multiple of 16, <= ATTN_TC_MAX_KEYS)
+  int32_t n_seg;       // own segments, one per pair the tile touches, in token order
+  int32_t pad;
+  // segment s: the pair starts at token tok_begin + (int16_t)(seg[s] & 0xffff) (<= 0 for
+  // a pair begun before the tile) and has seg[s] >> 16 tokens up to the tile's end
+  int32_t seg[ATTN_TC_MAX_SEGS];
 };
 
 struct Store {
@@ -234,12 +239,9 @@ cudaError_t launch_attention(const CUtensorMap& tm_pool, const AttnArgs& a, cuda
 // Arguments of the tensor-core attention kernel.
 struct AttnTcArgs {
   const AttnTile* tiles;
-  int n_units;             // tiles x kv heads
-  const int32_t* tok_off;  // sorted pair -> first packed token
-  int32_t tok0;            // first packed token of this chunk
+  int n_units;  // tiles x kv heads
   f16* out;
   int ld_out;
-  const int64_t* slot_row;
   int layer, Hq, Hkv;
   int* err;
 };
