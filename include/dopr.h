@@ -129,7 +129,10 @@ DOPR_API dopr_status dopr_store_create(const dopr_model_config *cfg, int64_t max
  *   m == 0 stores an empty prefix (the pass then equals a query-only forward).
  * The first put of a doc reserves its block; later puts must give the same
  * m (a different m is INVALID_ARG) and replace that layer.  A doc can be
- * scored once all n_layers layers were put.  Synchronous.
+ * scored once all n_layers layers were put.  The store keeps the values as
+ * fp16 (exact for bf16 values in fp16's normal range); a value that is not
+ * finite or exceeds 65504 in magnitude fails the put with INVALID_ARG and
+ * leaves that layer marked missing.  Synchronous.
  * Errors: INVALID_ARG, OUT_OF_MEMORY (pool full), CUDA.
  */
 DOPR_API dopr_status dopr_store_put(dopr_store *store, int64_t doc_id, int32_t m, int32_t layer, const void *k,
@@ -137,6 +140,39 @@ DOPR_API dopr_status dopr_store_put(dopr_store *store, int64_t doc_id, int32_t m
 
 /* Release a store.  NULL is accepted. */
 DOPR_API dopr_status dopr_store_destroy(dopr_store *store);
+
+/*
+ * Offline prefix construction (Sec. 3.3; Sec. 3.4's footnote): for each
+ * document d, forward its selected representations c_1..c_m (the compressed
+ * document inputs C~_d is built from) causally through the model as prefix
+ * inputs at positions 0..m-1, and store every layer's key (after the q/k
+ * norm and RoPE) and value as the document's prefix states -- the states
+ * dopr_store_put would be given.  The last layer stops after its key/value
+ * projection.
+ *   doc_ids   [n_docs] int64, host; distinct, each in [0, max_doc_id].
+ *   x_offsets [n_docs+1] int32, host: document d's representations are rows
+ *             x_offsets[d] .. x_offsets[d+1]-1 of x; x_offsets[0] == 0,
+ *             0 <= m_d <= 256 and m_d <= max_position.
+ *   x         bf16 [x_offsets[n_docs]][hidden]; a device pointer when
+ *             x_on_device != 0, else host memory (copied in by the call).
+ *   cuda_stream: a cudaStream_t, or NULL for the default stream.
+ * Documents are reserved (or must match an earlier reservation's m) before
+ * any kernel runs; on success every layer of every document is present.
+ * Synchronous.  Errors: INVALID_ARG, INCOMPLETE (model weights missing),
+ * OUT_OF_MEMORY (pool full), CUDA, TIMEOUT.
+ */
+DOPR_API dopr_status dopr_build_prefixes(dopr_model *model, dopr_store *store, int32_t n_docs, const int64_t *doc_ids,
+                                         const int32_t *x_offsets, const void *x, int32_t x_on_device,
+                                         void *cuda_stream);
+
+/*
+ * A stored layer of one document, read back for testing: k_out and v_out
+ * (host, fp16 bits [m][n_kv_heads][head_dim], the dopr_store_put layout).
+ * A document with m == 0 writes nothing.  Synchronous.
+ * Errors: INVALID_ARG, UNKNOWN_DOC (never stored), CUDA.
+ */
+DOPR_API dopr_status dopr_debug_store_read(const dopr_store *store, int64_t doc_id, int32_t layer, void *k_out,
+                                           void *v_out);
 
 /* Bytes of stored prefix state for one document of m prefix positions:
  * m * n_layers * 2 (K,V) * n_kv_heads * head_dim * 2 bytes.  This is the
@@ -243,7 +279,8 @@ DOPR_API dopr_status dopr_pack_order_noalloc(const dopr_store *store, int32_t n_
 /*
  * Per-kernel accounting, for measurement.  Every dopr_score call counts its
  * kernel launches per kernel family (pack, embed, gemm_qkv, qknorm_rope,
- * attention, gemm_o, rmsnorm, gemm_gate_up, gemm_down, score) together with
+ * attention, gemm_o, rmsnorm, gemm_gate_up, gemm_down, score, prefix_store;
+ * dopr_build_prefixes counts into the same families) together with
  * the algorithmic floating-point operations and device-memory bytes of those
  * launches (the minimum the operation needs: each input read once, each output
  * written once).  While enabled, each launch is also bracketed with CUDA

@@ -261,7 +261,7 @@ dopr_status map_device_error(int e) {
 }
 
 const char* kKindNames[K_COUNT] = {"pack", "embed", "gemm_qkv", "qknorm_rope", "attention",
-                                   "gemm_o", "rmsnorm", "gemm_gate_up", "gemm_down", "score"};
+                                   "gemm_o", "rmsnorm", "gemm_gate_up", "gemm_down", "score", "prefix_store"};
 
 // Launch `fn` as one kernel of family `kind`, counting it and, when profiling
 // is on, bracketing it with CUDA events on `st`.
@@ -482,7 +482,16 @@ dopr_status run_packer(Model* m, Store* s, int32_t n, const int32_t* dqo, const 
   return DOPR_OK;
 }
 
-dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cudaStream_t st) {
+// Prefix build mode of run_layers: the packed "tokens" are the selected document
+// representations (rows of x), each document one "pair" with no prefix and no score
+// token; after every layer's QKV projection its keys and values go to the store, and
+// the last layer stops there.
+struct BuildArgs {
+  const bf16* x;  // device, [total rows][hidden]
+};
+
+dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cudaStream_t st,
+                       const BuildArgs* build = nullptr) {
   Workspace& w = m->ws;
   const auto& c = m->cfg;
   const int H = c.hidden, F = c.ffn, L = c.n_layers, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
@@ -500,9 +509,10 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     double attn_keys = 0.0, prefix_rows = 0.0;
     for (int32_t sp = s0; sp < s1; ++sp) {
       const double Tp = w.h_tok_off[sp + 1] - w.h_tok_off[sp];
-      attn_keys += Tp * s->slot_m[w.h_sorted_slot[sp]] + Tp * (Tp + 1) / 2;
+      attn_keys += Tp * (build ? 0 : s->slot_m[w.h_sorted_slot[sp]]) + Tp * (Tp + 1) / 2;
     }
     for (int32_t it = plan.chunk_item[ci]; it < plan.chunk_item[ci + 1]; ++it) prefix_rows += w.h_items[it].m;
+    if (build) prefix_rows = 0.0;
     const double attn_flops = 4.0 * HEAD_DIM * Hq * attn_keys;
     const double attn_bytes = T * (2.0 * Hq + 2.0 * Hkv) * HEAD_DIM * 2 + prefix_rows * Hkv * 2 * HEAD_DIM * 2;
     // algorithmic bytes: operands once, outputs once (residual: read + write fp32, plus the next norm's bf16 operand)
@@ -511,7 +521,8 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     const auto gu = gemm_cost(T, 2.0 * F, H, T * F * 2.0);
     const auto dn = gemm_cost(T, H, F, T * H * 10.0);
     CUDA_TRY(prof_launch(m, K_EMBED_NORM, 1, 0.0, T * H * 8.0, st, [&] {
-      return launch_embed(w.tok_id + t0, Tc, m->embed, m->attn_norm, H, c.rms_eps, w.r, w.xn, w.ss_e, st);
+      return launch_embed(w.tok_id + t0, Tc, build ? build->x : m->embed, m->attn_norm, H, c.rms_eps, w.r, w.xn,
+                          w.ss_e, st);
     }));
     GemmParams base{};
     base.M = Tc;
@@ -571,6 +582,13 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       pq.k_cols = Hkv * HEAD_DIM;
       CUDA_TRY(prof_launch(m, K_GEMM_QKV, 1, qkv.first, qkv.second, st,
                            [&] { return launch_gemm(EPI_QKV, w.tm_xn, m->tm_qkv[l], pq, sms, st); }));
+      if (build) {  // this layer's keys and values are the document's stored prefix states
+        CUDA_TRY(prof_launch(m, K_PREFIX_STORE, 1, 0.0, T * 2.0 * Hkv * HEAD_DIM * 2 * 2, st, [&] {
+          return launch_prefix_store(w.qkv, m->qkv_dim, Tc, t0, Hq, Hkv, w.tok_pair, w.tok_pos, w.sorted_slot,
+                                     s->d_slot_row, s->d_slot_m, l, reinterpret_cast<f16*>(s->pool), st);
+        }));
+        if (last) continue;
+      }
       AttnArgs aa{};
       aa.items = w.items + (last ? plan.chunk_item[ci] : li0);
       aa.n_items = last ? plan.chunk_item[ci + 1] - plan.chunk_item[ci] : n_litems;
@@ -658,10 +676,56 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       CUDA_TRY(prof_launch(m, K_GEMM_DOWN, 1, last ? dn_last.first : dn.first, last ? dn_last.second : dn.second, st,
                            [&] { return launch_gemm(EPI_RESID_ADD, w.tm_act, m->tm_down[l], pd, sms, st); }));
     }
-    CUDA_TRY(prof_launch(m, K_SCORE, 1, 4.0 * H * (s1 - s0), (s1 - s0) * (H * 4.0 + 4.0), st, [&] {
-      return launch_score(w.r_s, H, w.tok_off, t0, s0, s1, 1, w.perm, m->final_norm, m->score_head, c.rms_eps,
-                          d_scores, st);
-    }));
+    if (!build) {
+      CUDA_TRY(prof_launch(m, K_SCORE, 1, 4.0 * H * (s1 - s0), (s1 - s0) * (H * 4.0 + 4.0), st, [&] {
+        return launch_score(w.r_s, H, w.tok_off, t0, s0, s1, 1, w.perm, m->final_norm, m->score_head, c.rms_eps,
+                            d_scores, st);
+      }));
+    }
+  }
+  return DOPR_OK;
+}
+
+// The slot of doc_id: reserved on its first use with prefix length m (a later use
+// must give the same m).  Host mirrors and device tables are updated together.
+dopr_status store_reserve(Store* s, int64_t doc_id, int32_t m, int32_t* slot_out) {
+  const auto& c = s->cfg;
+  int32_t slot = s->slot_of[doc_id];
+  if (slot >= 0 && s->slot_m[slot] != m)
+    return fail(DOPR_ERR_INVALID_ARG, "doc %lld was stored with m = %d, not %d", (long long)doc_id, s->slot_m[slot], m);
+  if (slot < 0) {
+    const int64_t need = 2 * (int64_t)c.n_kv_heads * m * c.n_layers;  // K and V rows of 128, every layer
+    if (s->used_rows + need > s->pool_rows)
+      return fail(DOPR_ERR_OUT_OF_MEMORY, "store pool full (%lld of %lld rows used, %lld needed)",
+                  (long long)s->used_rows, (long long)s->pool_rows, (long long)need);
+    slot = s->n_slots++;
+    s->slot_m.push_back(m);
+    s->slot_row.push_back(s->used_rows);
+    s->slot_layers.emplace_back(c.n_layers, 0);
+    s->slot_ok.push_back(0);
+    s->used_rows += need;
+    s->slot_of[doc_id] = slot;
+    const int64_t row = s->slot_row[slot];
+    CUDA_TRY(cudaMemcpy(s->d_slot_m + slot, &m, sizeof(int32_t), cudaMemcpyHostToDevice));
+    CUDA_TRY(cudaMemcpy(s->d_slot_row + slot, &row, sizeof(int64_t), cudaMemcpyHostToDevice));
+    CUDA_TRY(cudaMemcpy(s->d_slot_of + doc_id, &slot, sizeof(int32_t), cudaMemcpyHostToDevice));
+    s->max_m = std::max(s->max_m, m);
+  }
+  *slot_out = slot;
+  return DOPR_OK;
+}
+
+// Record that `layer` of `slot` holds valid states (present = 1) or not; the slot
+// becomes scoreable once every layer is present.
+dopr_status store_mark(Store* s, int32_t slot, int layer, bool present) {
+  const int L = s->cfg.n_layers;
+  s->slot_layers[slot][layer] = present ? 1 : 0;
+  bool all = true;
+  for (int l = 0; l < L; ++l) all = all && s->slot_layers[slot][l];
+  const uint8_t ok = all ? 1 : 0;
+  if (s->slot_ok[slot] != ok) {
+    s->slot_ok[slot] = ok;
+    CUDA_TRY(cudaMemcpy(s->d_slot_ok + slot, &ok, 1, cudaMemcpyHostToDevice));
   }
   return DOPR_OK;
 }
@@ -890,30 +954,11 @@ dopr_status dopr_store_put(dopr_store* s, int64_t doc_id, int32_t m, int32_t lay
   if (m < 0 || m > MAX_PREFIX) return fail(DOPR_ERR_INVALID_ARG, "m = %d outside [0, %d]", m, MAX_PREFIX);
   if (layer < 0 || layer >= c.n_layers) return fail(DOPR_ERR_INVALID_ARG, "bad layer %d", layer);
   if (m > 0 && (!k || !v)) return fail(DOPR_ERR_INVALID_ARG, "k or v is NULL");
-  int32_t slot = s->slot_of[doc_id];
-  if (slot >= 0 && s->slot_m[slot] != m)
-    return fail(DOPR_ERR_INVALID_ARG, "doc %lld was stored with m = %d, not %d", (long long)doc_id, s->slot_m[slot], m);
   const int64_t Hkv = c.n_kv_heads;
   const int64_t rows_per_layer = 2 * Hkv * m;  // K and V, [head][m] rows of 128
   CUDA_TRY(cudaSetDevice(s->device));
-  if (slot < 0) {
-    const int64_t need = rows_per_layer * c.n_layers;
-    if (s->used_rows + need > s->pool_rows)
-      return fail(DOPR_ERR_OUT_OF_MEMORY, "store pool full (%lld of %lld rows used, %lld needed)",
-                  (long long)s->used_rows, (long long)s->pool_rows, (long long)need);
-    slot = s->n_slots++;
-    s->slot_m.push_back(m);
-    s->slot_row.push_back(s->used_rows);
-    s->slot_layers.emplace_back(c.n_layers, 0);
-    s->slot_ok.push_back(0);
-    s->used_rows += need;
-    s->slot_of[doc_id] = slot;
-    const int64_t row = s->slot_row[slot];
-    CUDA_TRY(cudaMemcpy(s->d_slot_m + slot, &m, sizeof(int32_t), cudaMemcpyHostToDevice));
-    CUDA_TRY(cudaMemcpy(s->d_slot_row + slot, &row, sizeof(int64_t), cudaMemcpyHostToDevice));
-    CUDA_TRY(cudaMemcpy(s->d_slot_of + doc_id, &slot, sizeof(int32_t), cudaMemcpyHostToDevice));
-    s->max_m = std::max(s->max_m, m);
-  }
+  int32_t slot = -1;
+  STATUS_TRY(store_reserve(s, doc_id, m, &slot));
   if (m > 0) {
     const size_t bytes = (size_t)m * Hkv * HEAD_DIM * 2;
     f16* base = reinterpret_cast<f16*>(s->pool) + (size_t)(s->slot_row[slot] + layer * rows_per_layer) * HEAD_DIM;
@@ -939,26 +984,153 @@ dopr_status dopr_store_put(dopr_store* s, int64_t doc_id, int32_t m, int32_t lay
     if (e != cudaSuccess) return fail(DOPR_ERR_CUDA, "prefix store copy failed: %s", cudaGetErrorString(e));
     if (range) {
       // the layer now holds clamped data: mark it missing until a valid put replaces it
-      if (s->slot_layers[slot][layer] && s->slot_ok[slot]) {
-        s->slot_ok[slot] = 0;
-        const uint8_t zero = 0;
-        CUDA_TRY(cudaMemcpy(s->d_slot_ok + slot, &zero, 1, cudaMemcpyHostToDevice));
-      }
-      s->slot_layers[slot][layer] = 0;
+      STATUS_TRY(store_mark(s, slot, layer, false));
       return fail(DOPR_ERR_INVALID_ARG, "doc %lld layer %d: a prefix value is not finite or exceeds the fp16 range",
                   (long long)doc_id, layer);
     }
   }
-  if (!s->slot_layers[slot][layer]) {
-    s->slot_layers[slot][layer] = 1;
-    bool all = true;
-    for (int l = 0; l < c.n_layers; ++l) all = all && s->slot_layers[slot][l];
-    if (all) {
-      s->slot_ok[slot] = 1;
-      const uint8_t one = 1;
-      CUDA_TRY(cudaMemcpy(s->d_slot_ok + slot, &one, 1, cudaMemcpyHostToDevice));
-    }
+  return store_mark(s, slot, layer, true);
+}
+
+dopr_status dopr_build_prefixes(dopr_model* m, dopr_store* s, int32_t n_docs, const int64_t* doc_ids,
+                                const int32_t* x_offsets, const void* x, int32_t x_on_device, void* cuda_stream) {
+  g_last_error.clear();
+  STATUS_TRY(check_ready(m, s));
+  if (n_docs < 0) return fail(DOPR_ERR_INVALID_ARG, "n_docs < 0");
+  if (n_docs == 0) return DOPR_OK;
+  if (!doc_ids || !x_offsets) return fail(DOPR_ERR_INVALID_ARG, "NULL array");
+  const auto& c = m->cfg;
+  const int H = c.hidden, L = c.n_layers;
+  if (x_offsets[0] != 0) return fail(DOPR_ERR_INVALID_ARG, "x_offsets[0] must be 0");
+  std::vector<char> seen;
+  for (int32_t d = 0; d < n_docs; ++d) {
+    const int32_t md = x_offsets[d + 1] - x_offsets[d];
+    if (md < 0 || md > MAX_PREFIX) return fail(DOPR_ERR_INVALID_ARG, "doc %d: m = %d outside [0, %d]", d, md, MAX_PREFIX);
+    if (md > c.max_position) return fail(DOPR_ERR_INVALID_ARG, "doc %d: m = %d beyond max_position", d, md);
+    if (doc_ids[d] < 0 || doc_ids[d] > s->max_doc_id)
+      return fail(DOPR_ERR_INVALID_ARG, "doc_id %lld out of range", (long long)doc_ids[d]);
   }
+  {
+    std::vector<int64_t> ids(doc_ids, doc_ids + n_docs);
+    std::sort(ids.begin(), ids.end());
+    if (std::adjacent_find(ids.begin(), ids.end()) != ids.end())
+      return fail(DOPR_ERR_INVALID_ARG, "a doc_id appears twice in one build");
+  }
+  const int64_t rows = x_offsets[n_docs];
+  if (rows > 0 && !x) return fail(DOPR_ERR_INVALID_ARG, "x is NULL");
+  CUDA_TRY(cudaSetDevice(m->device));
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  Workspace& w = m->ws;
+  // slots first (validated above, so only a full pool can fail here)
+  std::vector<int32_t> slot(n_docs);
+  for (int32_t d = 0; d < n_docs; ++d) STATUS_TRY(store_reserve(s, doc_ids[d], x_offsets[d + 1] - x_offsets[d], &slot[d]));
+  // the documents with a prefix are the "pairs" of the pass, their rows its tokens
+  std::vector<int32_t> pd;
+  for (int32_t d = 0; d < n_docs; ++d)
+    if (x_offsets[d + 1] > x_offsets[d]) pd.push_back(d);
+  const int32_t n = (int32_t)pd.size();
+  if (n > 0) {
+    STATUS_TRY(ensure_call_buffers(m, n, rows, 0, 0));
+    std::vector<int32_t> tok_id(rows), tok_pos(rows), tok_pair(rows);
+    w.h_tok_off[0] = 0;
+    for (int32_t p = 0; p < n; ++p) {
+      const int32_t d = pd[p], md = x_offsets[d + 1] - x_offsets[d];
+      w.h_sorted_slot[p] = slot[d];
+      for (int32_t j = 0; j < md; ++j) {
+        const int32_t t = w.h_tok_off[p] + j;
+        tok_id[t] = x_offsets[d] + j;  // row of x (the embedding kernel gathers it)
+        tok_pos[t] = j;
+        tok_pair[t] = p;
+      }
+      w.h_tok_off[p + 1] = w.h_tok_off[p] + md;
+    }
+    const int64_t T = w.h_tok_off[n];
+    CUDA_TRY(cudaMemcpyAsync(w.tok_off, w.h_tok_off, sizeof(int32_t) * (n + 1), cudaMemcpyHostToDevice, st));
+    CUDA_TRY(cudaMemcpyAsync(w.sorted_slot, w.h_sorted_slot, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st));
+    CUDA_TRY(cudaMemcpyAsync(w.tok_id, tok_id.data(), sizeof(int32_t) * T, cudaMemcpyHostToDevice, st));
+    CUDA_TRY(cudaMemcpyAsync(w.tok_pos, tok_pos.data(), sizeof(int32_t) * T, cudaMemcpyHostToDevice, st));
+    CUDA_TRY(cudaMemcpyAsync(w.tok_pair, tok_pair.data(), sizeof(int32_t) * T, cudaMemcpyHostToDevice, st));
+    // chunks of whole documents; attention with no prefix, so a chunk's documents form one run
+    const int TT = attn_tc_rows_per_head(c.n_q_heads / c.n_kv_heads);
+    Plan plan;
+    plan.n_tokens = T;
+    plan.chunk_pair.assign(1, 0);
+    plan.chunk_item.assign(1, 0);
+    plan.chunk_litem.assign(1, 0);
+    plan.chunk_tile.assign(1, 0);
+    std::vector<AttnTile> tiles;
+    std::vector<AttnItem> litems;
+    for (int32_t s0 = 0; s0 < n;) {
+      int32_t s1 = s0 + 1;
+      while (s1 < n && w.h_tok_off[s1 + 1] - w.h_tok_off[s0] <= w.chunk_cap) ++s1;
+      plan_attention(w.h_tok_off, w.h_tok_off[s0], s0, s1, 0, 0, 0, TT, tiles, litems);
+      plan.chunk_pair.push_back(s1);
+      plan.chunk_item.push_back(0);
+      plan.chunk_litem.push_back((int32_t)litems.size());
+      plan.chunk_tile.push_back((int32_t)tiles.size());
+      s0 = s1;
+    }
+    plan.n_litems = (int32_t)litems.size();
+    plan.n_tiles = (int32_t)tiles.size();
+    if (plan.n_litems > w.item_cap || plan.n_litems > w.h_item_cap || plan.n_tiles > w.tile_cap)
+      return fail(DOPR_ERR_UNSUPPORTED, "attention plan exceeds its buffers");
+    std::copy(litems.begin(), litems.end(), w.h_items);
+    std::copy(tiles.begin(), tiles.end(), w.h_tiles);
+    if (plan.n_litems > 0)
+      CUDA_TRY(cudaMemcpyAsync(w.items, w.h_items, sizeof(AttnItem) * plan.n_litems, cudaMemcpyHostToDevice, st));
+    if (plan.n_tiles > 0)
+      CUDA_TRY(cudaMemcpyAsync(w.tiles, w.h_tiles, sizeof(AttnTile) * plan.n_tiles, cudaMemcpyHostToDevice, st));
+    // the representations on the device
+    const bf16* dx = static_cast<const bf16*>(x);
+    bf16* stage = nullptr;
+    if (!x_on_device) {
+      CUDA_TRY(cudaMalloc(&stage, sizeof(bf16) * (size_t)rows * H));
+      cudaError_t e = cudaMemcpyAsync(stage, x, sizeof(bf16) * (size_t)rows * H, cudaMemcpyHostToDevice, st);
+      if (e != cudaSuccess) {
+        cudaFree(stage);
+        return fail(DOPR_ERR_CUDA, "prefix input upload failed");
+      }
+      dx = stage;
+    }
+    CUDA_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), st));
+    BuildArgs b{dx};
+    const dopr_status rs = run_layers(m, s, plan, nullptr, st, &b);
+    cudaError_t e = cudaMemcpyAsync(w.h_err, w.err, sizeof(int), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (stage) cudaFree(stage);
+    STATUS_TRY(rs);
+    if (e != cudaSuccess) return fail(DOPR_ERR_CUDA, "prefix build failed: %s", cudaGetErrorString(e));
+    STATUS_TRY(map_device_error(*w.h_err));
+  }
+  for (int32_t d = 0; d < n_docs; ++d)
+    for (int l = 0; l < L; ++l) STATUS_TRY(store_mark(s, slot[d], l, true));
+  return DOPR_OK;
+}
+
+dopr_status dopr_debug_store_read(const dopr_store* s, int64_t doc_id, int32_t layer, void* k_out, void* v_out) {
+  g_last_error.clear();
+  if (!s) return fail(DOPR_ERR_INVALID_ARG, "store is NULL");
+  if (doc_id < 0 || doc_id > s->max_doc_id || s->slot_of[doc_id] < 0)
+    return fail(DOPR_ERR_UNKNOWN_DOC, "doc %lld is not stored", (long long)doc_id);
+  if (layer < 0 || layer >= s->cfg.n_layers) return fail(DOPR_ERR_INVALID_ARG, "bad layer %d", layer);
+  const int32_t slot = s->slot_of[doc_id], md = s->slot_m[slot];
+  const int Hkv = s->cfg.n_kv_heads;
+  if (md == 0) return DOPR_OK;
+  if (!k_out || !v_out) return fail(DOPR_ERR_INVALID_ARG, "NULL output");
+  CUDA_TRY(cudaSetDevice(s->device));
+  const size_t n = (size_t)2 * Hkv * md * HEAD_DIM;
+  std::vector<uint16_t> buf(n);
+  const uint16_t* src =
+      reinterpret_cast<const uint16_t*>(s->pool) + (size_t)(s->slot_row[slot] + (int64_t)layer * 2 * Hkv * md) * HEAD_DIM;
+  CUDA_TRY(cudaMemcpy(buf.data(), src, n * sizeof(uint16_t), cudaMemcpyDeviceToHost));
+  uint16_t* ko = static_cast<uint16_t*>(k_out);
+  uint16_t* vo = static_cast<uint16_t*>(v_out);
+  for (int g = 0; g < Hkv; ++g)  // pool [K|V][head][m][128] -> caller [m][head][128]
+    for (int j = 0; j < md; ++j)
+      for (int e = 0; e < HEAD_DIM; ++e) {
+        ko[((size_t)j * Hkv + g) * HEAD_DIM + e] = buf[((size_t)g * md + j) * HEAD_DIM + e];
+        vo[((size_t)j * Hkv + g) * HEAD_DIM + e] = buf[((size_t)(Hkv + g) * md + j) * HEAD_DIM + e];
+      }
   return DOPR_OK;
 }
 

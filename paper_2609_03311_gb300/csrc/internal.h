@@ -114,7 +114,7 @@ struct Workspace {
 // Per-kernel-family launch counters and (when enabled) CUDA-event timing.
 enum KernelKind : int {
   K_PACK = 0, K_EMBED_NORM, K_GEMM_QKV, K_QKNORM_ROPE, K_ATTENTION, K_GEMM_O, K_RMSNORM, K_GEMM_GATE_UP,
-  K_GEMM_DOWN, K_SCORE, K_COUNT
+  K_GEMM_DOWN, K_SCORE, K_PREFIX_STORE, K_COUNT
 };
 struct Profiler {
   bool on = false;
@@ -288,6 +288,10 @@ cudaError_t launch_pack_tokens(const PackArgs& a, cudaStream_t st);
 void set_last_error_message(const std::string& msg);
 
 // Debug kernel: bounded wait on a barrier nothing completes.
+// Prefix build: K/V rows of chunk tokens [0, T) (packed tokens t0 + t) into the store pool.
+cudaError_t launch_prefix_store(const f16* qkv, int ld_qkv, int T, int t0, int Hq, int Hkv, const int32_t* tok_pair,
+                                const int32_t* tok_pos, const int32_t* pair_slot, const int64_t* slot_row,
+                                const int32_t* slot_m, int layer, f16* pool, cudaStream_t st);
 cudaError_t launch_wait_timeout_probe(int* err, uint64_t timeout_ns, cudaStream_t st);
 
 }  // namespace dopr

@@ -139,6 +139,27 @@ __global__ void k_store_transpose(const uint4* __restrict__ k, const uint4* __re
   if (bad) atomicOr(range, 1);
 }
 
+// Prefix build (Sec. 3.3): copy each token's key (after the q/k norm and RoPE) and
+// raw value of every kv head from the packed QKV buffer into its document's block of
+// the store pool, in the layout dopr_store_put writes: per layer, K then V, per kv
+// head, m rows of 128.  One warp per (token, kv head, K|V), 8 bytes a lane.
+__global__ void k_prefix_store(const f16* __restrict__ qkv, int ld_qkv, int T, int t0, int Hq, int Hkv,
+                               const int32_t* __restrict__ tok_pair, const int32_t* __restrict__ tok_pos,
+                               const int32_t* __restrict__ pair_slot, const int64_t* __restrict__ slot_row,
+                               const int32_t* __restrict__ slot_m, int layer, f16* __restrict__ pool) {
+  const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (w >= static_cast<int64_t>(T) * Hkv * 2) return;
+  const int kv = static_cast<int>(w & 1);
+  const int g = static_cast<int>((w >> 1) % Hkv);
+  const int t = static_cast<int>((w >> 1) / Hkv);
+  const int p = tok_pair[t0 + t], j = tok_pos[t0 + t];
+  const int slot = pair_slot[p];
+  const int64_t row = slot_row[slot] + (static_cast<int64_t>(layer * 2 + kv) * Hkv + g) * slot_m[slot] + j;
+  const uint2* src = reinterpret_cast<const uint2*>(qkv + static_cast<int64_t>(t) * ld_qkv + (Hq + kv * Hkv + g) * HEAD_DIM);
+  reinterpret_cast<uint2*>(pool + row * HEAD_DIM)[lane] = src[lane];
+}
+
 // Test kernel: one bounded wait on an mbarrier that is never completed.
 __global__ void k_wait_timeout_probe(int* err, uint64_t timeout_ns) {
   __shared__ uint64_t bar;
@@ -195,6 +216,16 @@ cudaError_t launch_store_transpose(const bf16* k, const bf16* v, int m, int Hkv,
   const int blocks = static_cast<int>((n + 255) / 256);
   k_store_transpose<<<blocks, 256, 0, st>>>(reinterpret_cast<const uint4*>(k), reinterpret_cast<const uint4*>(v), m,
                                             Hkv, reinterpret_cast<uint4*>(dk), reinterpret_cast<uint4*>(dv), range);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prefix_store(const f16* qkv, int ld_qkv, int T, int t0, int Hq, int Hkv, const int32_t* tok_pair,
+                                const int32_t* tok_pos, const int32_t* pair_slot, const int64_t* slot_row,
+                                const int32_t* slot_m, int layer, f16* pool, cudaStream_t st) {
+  const int64_t threads = static_cast<int64_t>(T) * Hkv * 2 * 32;
+  if (threads <= 0) return cudaSuccess;
+  k_prefix_store<<<static_cast<unsigned>((threads + 255) / 256), 256, 0, st>>>(
+      qkv, ld_qkv, T, t0, Hq, Hkv, tok_pair, tok_pos, pair_slot, slot_row, slot_m, layer, pool);
   return cudaGetLastError();
 }
 

@@ -73,6 +73,8 @@ def load():
         "dopr_pack_order_noalloc": ([P, i32, P, P, P, P, P], i32),
         "dopr_profile_enable": ([P, i32], i32),
         "dopr_profile_read": ([P, P, i32], i32),
+        "dopr_build_prefixes": ([P, P, i32, P, P, P, i32, P], i32),
+        "dopr_debug_store_read": ([P, i64, i32, P, P], i32),
         "dopr_last_error": ([], ctypes.c_char_p),
         "dopr_version": ([], ctypes.c_char_p),
     }
@@ -184,6 +186,13 @@ class Store:
         for l in range(k.shape[0]):
             self.put_layer(doc_id, l, k[l], v[l])
 
+    def read_layer(self, doc_id: int, layer: int, m: int):
+        """The stored (fp16) K and V of one layer as float16 [m, n_kv_heads, 128] numpy arrays."""
+        shape = (m, self.cfg.n_kv_heads, self.cfg.head_dim)
+        k, v = np.zeros(shape, np.float16), np.zeros(shape, np.float16)
+        _check(load().dopr_debug_store_read(self._h, int(doc_id), int(layer), k.ctypes.data, v.ctypes.data))
+        return k, v
+
     def close(self):
         if self._h:
             load().dopr_store_destroy(self._h)
@@ -194,6 +203,19 @@ class Store:
             self.close()
         except Exception:
             pass
+
+
+def build_prefixes(model: Model, store: Store, doc_ids, x_offsets, x: torch.Tensor, stream=None):
+    """Offline prefix construction: forward each document's representations
+    x[x_offsets[d]:x_offsets[d+1]] (bf16 [rows, hidden], on the GPU or the host)
+    and store every layer's keys and values for doc_ids[d]."""
+    di, xo = _host(doc_ids, np.int64), _host(x_offsets, np.int32)
+    assert x.dtype == torch.bfloat16 and x.dim() == 2
+    x = x.contiguous()
+    st = ctypes.c_void_p(stream.cuda_stream if stream is not None else
+                         (torch.cuda.current_stream().cuda_stream if x.is_cuda else 0))
+    _check(load().dopr_build_prefixes(model._h, store._h, len(di), di.ctypes.data, xo.ctypes.data, _ptr(x),
+                                      int(x.is_cuda), st))
 
 
 def score(model: Model, store: Store, q_offsets, q_tokens, doc_ids, out=None, stream=None) -> torch.Tensor:

@@ -178,6 +178,18 @@ def make_prefix(shape: ModelShape, m: int, doc: int, seed: int = 0, device="cpu"
     return k, v
 
 
+def make_doc_representations(shape: ModelShape, doc_m: dict, seed: int = 0, device="cpu"):
+    """Selected document representations c_1..c_m per document (the prefix
+    inputs of offline prefix construction): bf16 rows ~ N(0,1) of width hidden,
+    documents in sorted doc-id order.  Returns (doc_ids int64, x_offsets int32
+    [n+1], x bf16 [sum m, hidden])."""
+    docs = sorted(doc_m)
+    offs = np.concatenate([[0], np.cumsum([doc_m[d] for d in docs])]).astype(np.int32)
+    parts = [_normal_bf16((doc_m[d], shape.hidden), 1.0, device, seed, "doc_repr", d) for d in docs]
+    x = torch.cat(parts) if parts else torch.zeros((0, shape.hidden), dtype=torch.bfloat16, device=device)
+    return np.asarray(docs, dtype=np.int64), offs, x
+
+
 def make_prefix_batch(shape: ModelShape, m: int, docs, seed: int = 0, device="cpu"):
     """Prefix states for many documents of the same m in one draw per doc
     group: K, V bf16 [n_docs, L, m, Hkv, D].  The sub-stream is keyed by
