@@ -227,8 +227,9 @@ def setup(wl, seed, device, need_host_weights):
 
 
 def gemm_traffic_record():
-    """ncu-measured DRAM traffic per GEMM launch, valid only for the kernel
-    source it was captured from (else None)."""
+    """ncu-measured DRAM traffic of the projection GEMMs as a multiple of their
+    algorithmic bytes, valid only for the kernel source it was captured from
+    (else None)."""
     path = os.path.join(ROOT, "profiles", "gemm_traffic.json")
     if not os.path.exists(path):
         return None
@@ -372,7 +373,7 @@ def run_dopr(args, rank, world, local_rank, dist):
                 "achieved": achieved, "peak": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s",
                 "frac": (achieved / peaks["bf16_tflops_sustained"]) if achieved else None,
                 "peak_source": f"{peaks['source']} sustained bf16 (kernel timed inside a long step)",
-                "traffic": (traffic["dram_bytes_per_launch"] if traffic else None),
+                "traffic": (traffic["traffic_over_algorithmic"] * g_bytes / max(g_launch, 1) if traffic else None),
                 "algorithmic_flops_per_launch": g_flops / max(g_launch, 1),
                 "algorithmic_bytes_per_launch": g_bytes / max(g_launch, 1),
                 "share_of_step": g_ms / tot_ms}
