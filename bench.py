@@ -51,6 +51,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--latency-queries", type=int, default=10)
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--reuse", action="store_true",
+                    help="amortised cost under document reuse (T_off, T_full, T_online, Speedup(r)) instead of the bench")
     return ap.parse_args()
 
 
@@ -431,6 +433,85 @@ def run_dopr(args, rank, world, local_rank, dist):
         print(json.dumps(line))
 
 
+def run_reuse(args):
+    """Controlled cross-query reuse (the paper's amortised speedup): one document
+    scored for r queries costs r * T_full uncompressed and T_off + r * T_online with
+    DoPR, Speedup(r) = r T_full / (T_off + r T_online).  Measured on the workload's
+    model: T_online per pair on its compressed prefixes, T_full per pair on
+    [document tokens ; query ; t_score] with no prefix, and T_off per document =
+    a document-only forward over its tokens (where the salient positions would be
+    read) + the prefix build over its m selected representations."""
+    import torch
+
+    from paper_2609_03311_gb300 import dopr, synth
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    wl = synth.WORKLOADS[args.workload]
+    full_wl = synth.WORKLOADS["qwen3-8b-fulldoc"] if wl.model.name == "qwen3-8b" else wl
+    n_doc_tokens = full_wl.fulldoc_tokens or 512
+    cfg, model, store, doc_m, _ = setup(wl, args.seed, dev, False)
+    s = wl.model
+    empty = dopr.Store(cfg, wl.n_docs - 1, 1 << 16)  # every document with m = 0
+    for d in range(wl.n_docs):
+        z = torch.zeros((s.n_layers, 0, s.n_kv_heads, s.head_dim), dtype=torch.bfloat16)
+        empty.put(d, z, z)
+    pairs = synth.make_workload_pairs(wl, seed=args.seed)
+    per_q = wl.docs_per_query
+
+    def timed(fn, reps):
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            fn()
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        return statistics.median(ts)
+
+    def dev_batch(b):
+        return (torch.tensor(b["q_offsets"], device=dev), torch.tensor(b["q_tokens"], device=dev),
+                torch.tensor(b["doc_ids"], device=dev))
+
+    # T_online: 20 queries' candidate lists against the compressed prefixes
+    n_on = 20 * per_q
+    on = dev_batch(slice_pairs(pairs, 0, n_on))
+    t_online = timed(lambda: dopr.score(model, store, *on), args.steps) / n_on
+    # T_full: 2 queries' lists as [document tokens ; query]
+    n_full = 2 * per_q
+    full_pairs = build_pairs(full_wl, args.seed) if full_wl is not wl else None
+    if full_pairs is None:
+        raise SystemExit("--reuse needs the 8B workload family")
+    fb = dev_batch(slice_pairs(full_pairs, 0, n_full))
+    t_full = timed(lambda: dopr.score(model, empty, *fb), max(1, args.steps // 2)) / n_full
+    # T_off: the document-only forward over 100 documents' tokens, then the prefix build of their m rows
+    docs = np.arange(100, dtype=np.int64)
+    toks = [synth.make_fulldoc_tokens(full_wl, int(d), seed=args.seed) for d in docs]
+    qo = np.concatenate([[0], np.cumsum([len(t) for t in toks])]).astype(np.int32)
+    doc_pass = (torch.tensor(qo, device=dev), torch.tensor(np.concatenate(toks), device=dev),
+                torch.tensor(docs, device=dev))
+    t_doc = timed(lambda: dopr.score(model, empty, *doc_pass), args.steps) / len(docs)
+    m = int(doc_m[0])
+    bstore = dopr.Store(cfg, len(docs) - 1, len(docs) * dopr.prefix_bytes(cfg, m))
+    ids, offs, x = synth.make_doc_representations(s, {int(d): m for d in docs}, seed=args.seed, device=dev)
+    t_build = timed(lambda: dopr.build_prefixes(model, bstore, ids, offs, x), args.steps) / len(docs)
+    t_off = t_doc + t_build
+    rs = [1, 2, 4, 8, 16, 32, 64, 128]
+    print(json.dumps({
+        "metric": "amortised speedup under document reuse, r T_full / (T_off + r T_online)", "unit": "x",
+        "config": {"workload": wl.name, "model": s.name, "m": m, "document_tokens": n_doc_tokens,
+                   "online_pairs": n_on, "full_pairs": n_full, "offline_documents": len(docs)},
+        "t_online_ms_per_pair": t_online, "t_full_ms_per_pair": t_full,
+        "t_off_ms_per_doc": t_off, "t_off_parts_ms": {"document_forward": t_doc, "prefix_build": t_build},
+        "speedup": {str(r): r * t_full / (t_off + r * t_online) for r in rs},
+        "speedup_limit": t_full / t_online, "data": "synthetic", "dtype": "f16",
+    }))
+
+
 def run_reference(args, rank, world):
     """The oracle alone, on the host cores, on bounded samples of the workload."""
     if rank != 0:
@@ -483,7 +564,9 @@ def main():
             torch.cuda.set_device(local_rank)
         tdist.init_process_group(backend=backend)
         dist = tdist
-    if args.impl == "reference":
+    if args.reuse:
+        run_reuse(args)
+    elif args.impl == "reference":
         run_reference(args, rank, world)
     else:
         run_dopr(args, rank, world, local_rank, dist)
