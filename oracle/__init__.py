@@ -72,7 +72,10 @@ def load(lib_path: str | None = None):
     lib.oracle_attend.argtypes = [P, P, P, ctypes.c_int, ctypes.c_int, f64, P]
     lib.oracle_silu.argtypes = [f64]
     lib.oracle_silu.restype = f64
-    lib.oracle_forward.argtypes = [P, ctypes.c_int, P, ctypes.c_int, ctypes.c_int, P, P, P, P, P, P]
+    lib.oracle_forward.argtypes = [P, ctypes.c_int, P, ctypes.c_int, ctypes.c_int, P, P, P, P, P, P, P]
+    lib.oracle_attn_probs.argtypes = [P, P, ctypes.c_int, ctypes.c_int, f64, P]
+    lib.oracle_salience.argtypes = [ctypes.c_int, P, ctypes.c_int, P]
+    lib.oracle_select_topk.argtypes = [ctypes.c_int, P, ctypes.c_int, P]
     lib.oracle_score_head.argtypes = [P, P]
     lib.oracle_score_head.restype = f64
     lib.oracle_embed.argtypes = [P, ctypes.c_int, P, P]
@@ -154,6 +157,7 @@ class OracleModel:
             return u.ctypes.data
 
         m.embed = hold(weights["embed"])
+        self._final_norm = bf16_to_f64(weights["final_norm"])
         m.final_norm = hold(weights["final_norm"])
         m.score_head = hold(weights["score_head"])
         for name in self._PER_LAYER:
@@ -175,10 +179,12 @@ class OracleModel:
             raise ValueError(f"oracle_embed rc={rc}")
         return x
 
-    def forward(self, x0, pos0: int, prefix_k=None, prefix_v=None, want_kv=False, want_attn=False):
+    def forward(self, x0, pos0: int, prefix_k=None, prefix_v=None, want_kv=False, want_attn=False,
+                want_probs=False):
         """Causal pass over online vectors x0 [T,H] at positions pos0..;
         prefix_k/v: [L,m,Hkv,D] fp64 or None.  Returns dict with 'h' and
-        optionally 'k', 'v' ([L,T,Hkv,D]) and 'attn' ([L,T,Hq*D])."""
+        optionally 'k', 'v' ([L,T,Hkv,D]), 'attn' ([L,T,Hq*D]) and 'probs'
+        ([T, m+T], the last layer's head-averaged attention weights)."""
         s = self.shape
         x0 = _f64(x0)
         T = x0.shape[0]
@@ -189,8 +195,9 @@ class OracleModel:
         k = np.zeros((s.n_layers, T, s.n_kv_heads, s.head_dim)) if want_kv else None
         v = np.zeros_like(k) if want_kv else None
         a = np.zeros((s.n_layers, T, s.n_q_heads * s.head_dim)) if want_attn else None
+        pr = np.zeros((T, m + T)) if want_probs else None
         rc = self.lib.oracle_forward(self.ref, T, _ptr(x0), int(pos0), m, _ptr(pk), _ptr(pv),
-                                     _ptr(h), _ptr(k), _ptr(v), _ptr(a))
+                                     _ptr(h), _ptr(k), _ptr(v), _ptr(a), _ptr(pr))
         if rc != 0:
             raise ValueError(f"oracle_forward rc={rc}")
         out = {"h": h}
@@ -198,7 +205,25 @@ class OracleModel:
             out["k"], out["v"] = k, v
         if want_attn:
             out["attn"] = a
+        if want_probs:
+            out["probs"] = pr
         return out
+
+    def select(self, ids, top_k: int, top_p: int):
+        """Attention-based key token selection (Sec. 3.2.1) for one document of
+        token ids: encode it alone at positions 0..n-1, salience u from the last
+        layer's head-averaged attention, the top_k positions (ascending), and
+        their final-layer states (after the final RMSNorm).
+        Returns (u [n], positions [k], states [k, H])."""
+        x = self.embed(ids)
+        out = self.forward(x, 0, want_probs=True)
+        n = len(ids)
+        u = salience(out["probs"], top_p)
+        pos = select_topk(u, top_k)
+        g = self._final_norm
+        states = np.stack([rmsnorm(out["h"][i], g, self.shape.rms_eps) for i in pos]) if len(pos) else \
+            np.zeros((0, self.shape.hidden))
+        return u, pos, states
 
     def score_head(self, h) -> float:
         h = _f64(h)
@@ -255,6 +280,35 @@ def attend(q, K, V, scale) -> np.ndarray:
     out = np.zeros(q.size)
     lib.oracle_attend(_ptr(q), _ptr(K), _ptr(V), K.shape[0], q.size, float(scale), _ptr(out))
     return out
+
+
+def attn_probs(q, K, scale) -> np.ndarray:
+    q, K = _f64(q), _f64(K)
+    n, D = K.shape
+    p = np.zeros(n)
+    load().oracle_attn_probs(_ptr(q), _ptr(K), n, D, float(scale), _ptr(p))
+    return p
+
+
+def salience(A, top_p: int) -> np.ndarray:
+    """Column top-p means of a causal [n, n] attention matrix (Sec. 3.2.1)."""
+    A = _f64(A)
+    n = A.shape[0]
+    u = np.zeros(n)
+    rc = load().oracle_salience(n, _ptr(A), int(top_p), _ptr(u))
+    if rc != 0:
+        raise ValueError(f"oracle_salience rc={rc}")
+    return u
+
+
+def select_topk(u, K: int) -> np.ndarray:
+    """Ascending positions of the K largest u (ties to the lower position)."""
+    u = _f64(u)
+    idx = np.zeros(max(len(u), 1), dtype=np.int32)
+    k = load().oracle_select_topk(len(u), _ptr(u), int(K), _ptr(idx))
+    if k < 0:
+        raise ValueError("oracle_select_topk failed")
+    return idx[:k]
 
 
 def silu(x: float) -> float:

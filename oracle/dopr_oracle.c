@@ -29,6 +29,12 @@
  *   - RMSNorm(x) = x / sqrt(mean(x^2) + eps) * g;
  *   - score = <W_s[0], RMSNorm(h_last) * g_final> - <W_s[1], ...>.
  *
+ * Also here: the attention-based key token selection of Sec. 3.2.1 (the
+ * last layer's head-averaged attention weights from oracle_forward, the
+ * column top-p salience, the top-K positions), which the offline prefix
+ * construction feeds from.  The paper leaves p open; ties in the ranking go to
+ * the lower position and the selected positions come out in ascending order.
+ *
  * Everything is fp64.  Weights and stored states arrive as bf16 bit
  * patterns (uint16) or fp64 and are widened exactly; no intermediate value
  * is rounded.  Parallelism (OpenMP) is only over independent outputs (one
@@ -132,6 +138,23 @@ void oracle_attend(const double *q, const double *K, const double *V, int n, int
     free(s);
 }
 
+/* The softmax weights themselves: p[i] = exp(s_i - max) / sum_j exp(s_j - max),
+ * s_i = <q, K_i> * scale, i < n (the weights oracle_attend applies to V). */
+void oracle_attn_probs(const double *q, const double *K, int n, int D, double scale, double *p)
+{
+    if (n <= 0) return;
+    double mx = -INFINITY;
+    for (int i = 0; i < n; ++i) {
+        double acc = 0.0;
+        for (int d = 0; d < D; ++d) acc += q[d] * K[(size_t)i * D + d];
+        p[i] = acc * scale;
+        if (p[i] > mx) mx = p[i];
+    }
+    double z = 0.0;
+    for (int i = 0; i < n; ++i) { p[i] = exp(p[i] - mx); z += p[i]; }
+    for (int i = 0; i < n; ++i) p[i] /= z;
+}
+
 double oracle_silu(double x) { return x / (1.0 + exp(-x)); }
 
 /* Y[t][o] = sum_i X[t][i] * W[o][i] for t < T, o < out; W is bf16. */
@@ -171,10 +194,14 @@ static void widen(const uint16_t *src, int n, double *dst)
  *   k_out   [L][T][Hkv][D]    keys the online tokens produced (post norm+RoPE)
  *   v_out   [L][T][Hkv][D]    values the online tokens produced
  *   attn_out[L][T][Hq*D]      attention outputs before the output projection
+ *   probs_out[T][m+T]         the last layer's attention weights averaged over
+ *                             the q heads (row = attending token, column = key:
+ *                             prefix slots, then online tokens; 0 where masked) --
+ *                             the matrix A-bar of Sec. 3.2.1 when m == 0
  */
 int oracle_forward(const oracle_model *M, int T, const double *x0, int pos0, int m,
                    const double *pk, const double *pv, double *h_out, double *k_out,
-                   double *v_out, double *attn_out)
+                   double *v_out, double *attn_out, double *probs_out)
 {
     if (!M || T < 0 || m < 0 || !h_out || (T > 0 && !x0) || (m > 0 && (!pk || !pv)))
         return ORACLE_ERR_ARG;
@@ -252,6 +279,25 @@ int oracle_forward(const oracle_model *M, int T, const double *x0, int pos0, int
                               att + ((size_t)t * Hq + h) * D);
             }
         if (attn_out) memcpy(attn_out + (size_t)l * T * Hq * D, att, sizeof(double) * (size_t)T * Hq * D);
+        if (probs_out && l == L - 1) {
+            /* head average of the last layer's weights, heads added in index order */
+            #pragma omp parallel
+            {
+                double *pw = (double *)malloc(sizeof(double) * (size_t)S);
+                #pragma omp for schedule(static)
+                for (int t = 0; t < T; ++t) {
+                    double *row = probs_out + (size_t)t * S;
+                    for (int i = 0; i < S; ++i) row[i] = 0.0;
+                    for (int h = 0; h < Hq; ++h) {
+                        const int kvh = h / G;
+                        oracle_attn_probs(q + ((size_t)t * Hq + h) * D, Kall + (size_t)kvh * S * D, m + t + 1, D,
+                                          scale, pw);
+                        for (int i = 0; i <= m + t; ++i) row[i] += pw[i] / (double)Hq;
+                    }
+                }
+                free(pw);
+            }
+        }
         /* output projection + residual */
         linear_bf16(att, T, Hq * D, M->wo[l], H, dlt);
         for (size_t i = 0; i < (size_t)T * H; ++i) r[i] += dlt[i];
@@ -330,12 +376,77 @@ int oracle_score_pairs(const oracle_model *M, int n_pairs, const int32_t *q_offs
         }
         if (rc == ORACLE_OK)
             rc = oracle_forward(M, T, x, m, m, m > 0 ? doc_k[d] : NULL, m > 0 ? doc_v[d] : NULL,
-                                h, NULL, NULL, NULL);
+                                h, NULL, NULL, NULL, NULL);
         if (rc == ORACLE_OK) scores[p] = oracle_score_head(M, h + (size_t)(T - 1) * H);
         free(ids); free(x); free(h);
         if (rc != ORACLE_OK) return rc;
     }
     return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------ */
+/* Attention-based key token selection (Sec. 3.2.1)                   */
+
+static int cmp_desc(const void *a, const void *b)
+{
+    const double x = *(const double *)a, y = *(const double *)b;
+    return (x < y) - (x > y);
+}
+
+/*
+ * Salience of each document token from the head-averaged final-layer
+ * attention matrix A[n][n] (row = attending token, causal: A[t][i] = 0 for
+ * i > t): u_i = the mean of the top_p largest values of column i among its
+ * n - i causal entries A[i..n-1][i], i.e. of min(top_p, n - i) values
+ * (0-based i; the paper's 1-based min(p, n - i + 1)).
+ */
+int oracle_salience(int n, const double *A, int top_p, double *u)
+{
+    if (n < 0 || top_p < 1 || (n > 0 && (!A || !u))) return ORACLE_ERR_ARG;
+    double *col = (double *)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+    if (!col) return ORACLE_ERR_NOMEM;
+    for (int i = 0; i < n; ++i) {
+        const int cnt = n - i;
+        for (int t = i; t < n; ++t) col[t - i] = A[(size_t)t * n + i];
+        qsort(col, (size_t)cnt, sizeof(double), cmp_desc);
+        const int k = top_p < cnt ? top_p : cnt;
+        double acc = 0.0;
+        for (int j = 0; j < k; ++j) acc += col[j];
+        u[i] = acc / (double)k;
+    }
+    free(col);
+    return ORACLE_OK;
+}
+
+typedef struct { double u; int32_t idx; } sal_key;
+
+static int cmp_sal(const void *a, const void *b)
+{
+    const sal_key *x = (const sal_key *)a, *y = (const sal_key *)b;
+    if (x->u != y->u) return (x->u < y->u) - (x->u > y->u); /* larger salience first */
+    return (x->idx > y->idx) - (x->idx < y->idx);          /* then the lower index  */
+}
+
+static int cmp_i32(const void *a, const void *b)
+{
+    const int32_t x = *(const int32_t *)a, y = *(const int32_t *)b;
+    return (x > y) - (x < y);
+}
+
+/* The positions of the k most salient tokens (k = min(K, n)), equal salience
+ * going to the lower position, written in ascending position order; returns k. */
+int oracle_select_topk(int n, const double *u, int K, int32_t *idx)
+{
+    if (n < 0 || K < 0 || (n > 0 && (!u || !idx))) return -1;
+    const int k = K < n ? K : n;
+    sal_key *keys = (sal_key *)malloc(sizeof(sal_key) * (size_t)(n > 0 ? n : 1));
+    if (!keys) return -1;
+    for (int i = 0; i < n; ++i) { keys[i].u = u[i]; keys[i].idx = i; }
+    qsort(keys, (size_t)n, sizeof(sal_key), cmp_sal);
+    for (int j = 0; j < k; ++j) idx[j] = keys[j].idx;
+    qsort(idx, (size_t)k, sizeof(int32_t), cmp_i32);
+    free(keys);
+    return k;
 }
 
 /* ------------------------------------------------------------------ */

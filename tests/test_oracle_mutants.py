@@ -41,6 +41,10 @@ MUTANTS = [
     ("stored_v_from_k", "const double *sv = pv + (((size_t)l * m + i) * Hkv + g) * D;",
      "const double *sv = pk + (((size_t)l * m + i) * Hkv + g) * D;"),
     ("pack_positions_unshifted", "tok_pos[off + j] = pair_m[p] + j;", "tok_pos[off + j] = j;"),
+    ("salience_mean_over_all", "u[i] = acc / (double)k;", "u[i] = acc / (double)cnt;"),
+    ("topk_ties_to_higher", "return (x->idx > y->idx) - (x->idx < y->idx);", "return (x->idx < y->idx) - (x->idx > y->idx);"),
+    ("probs_average_over_kv_heads", "row[i] += pw[i] / (double)Hq;", "row[i] += pw[i] / (double)Hkv;"),
+    ("probs_key_count", "Kall + (size_t)kvh * S * D, m + t + 1, D,", "Kall + (size_t)kvh * S * D, m + t, D,"),
 ]
 
 

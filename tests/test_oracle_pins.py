@@ -315,3 +315,65 @@ def test_pack_plan_against_python_stable_sort():
                 assert plan["tok_pair"][off + j] == s
             off += L + 1
         assert plan["tok_off"][n] == off
+
+
+# --------------------------------------------- key token selection (Sec. 3.2.1)
+
+def test_salience_hand_worked_matrix():
+    # column i's causal entries are rows i..n-1; u_i = mean of the top-p of them
+    A = np.array([[1.0, 0.0, 0.0, 0.0],
+                  [0.25, 0.75, 0.0, 0.0],
+                  [0.5, 0.2, 0.3, 0.0],
+                  [0.1, 0.6, 0.1, 0.2]])
+    np.testing.assert_allclose(oracle.salience(A, 1), [1.0, 0.75, 0.3, 0.2], rtol=0, atol=1e-15)
+    np.testing.assert_allclose(oracle.salience(A, 2), [0.75, 0.675, 0.2, 0.2], rtol=0, atol=1e-15)
+    np.testing.assert_allclose(oracle.salience(A, 4), [1.85 / 4, 1.55 / 3, 0.4 / 2, 0.2], rtol=0, atol=1e-15)
+    np.testing.assert_allclose(oracle.salience(A, 100), oracle.salience(A, 4), rtol=0, atol=0)
+
+
+def test_select_topk_against_brute_force_with_ties():
+    rng = np.random.default_rng(3)
+    for n, K in ((1, 1), (7, 3), (40, 40), (40, 55), (200, 16)):
+        u = rng.integers(0, 6, size=n).astype(np.float64) / 5.0  # many exact ties
+        want = sorted(sorted(range(n), key=lambda i: (-u[i], i))[:min(K, n)])
+        np.testing.assert_array_equal(oracle.select_topk(u, K), want)
+
+
+def test_attention_weights_uniform_when_wq_zero():
+    # W_q = 0 => every causal key of token t weighs 1/(t+1) in every head, so the
+    # head-averaged matrix is A[t][i] = 1/(t+1) for i <= t; column i's top-p are
+    # 1/(i+1) .. 1/(i+k), k = min(p, n - i).
+    om, w = tiny_model(seed=8, zero=("wq",))
+    rng = np.random.default_rng(8)
+    n = 9
+    out = om.forward(om.embed(rng.integers(0, TINY.vocab, size=n)), 0, want_probs=True)
+    want = np.tril(np.ones((n, n))) / np.arange(1, n + 1)[:, None]
+    np.testing.assert_allclose(out["probs"], want, rtol=1e-13, atol=1e-15)
+    for p in (1, 3, n):
+        u = oracle.salience(out["probs"], p)
+        for i in range(n):
+            k = min(p, n - i)
+            assert abs(u[i] - np.mean(1.0 / np.arange(i + 1, i + k + 1))) <= 1e-13
+
+
+def test_attention_weights_rows_causal_and_consistent_with_outputs():
+    # rows sum to 1, nothing above the diagonal (beyond the prefix); with one kv head
+    # the head-averaged weights applied to the last layer's values give the mean of
+    # the heads' attention outputs (oracle_attend's own path).
+    shape = synth.ModelShape("tiny-kv1", n_layers=2, hidden=64, n_q_heads=4, n_kv_heads=1, head_dim=16, ffn=96,
+                             vocab=50, rope_theta=1e4, rms_eps=1e-6)
+    om, _ = tiny_model(seed=9, shape=shape)
+    rng = np.random.default_rng(9)
+    m, T = 3, 8
+    pk = rng.normal(size=(shape.n_layers, m, 1, shape.head_dim))
+    pv = rng.normal(size=(shape.n_layers, m, 1, shape.head_dim))
+    out = om.forward(om.embed(rng.integers(0, shape.vocab, size=T)), m, pk, pv, want_kv=True, want_attn=True,
+                     want_probs=True)
+    P = out["probs"]
+    np.testing.assert_allclose(P.sum(1), 1.0, rtol=0, atol=1e-13)
+    for t in range(T):
+        assert np.all(P[t, m + t + 1:] == 0.0)
+    L, D = shape.n_layers - 1, shape.head_dim
+    V = np.concatenate([pv[L, :, 0], out["v"][L, :, 0]], 0)  # [m + T, D]
+    head_mean = out["attn"][L].reshape(T, shape.n_q_heads, D).mean(1)
+    np.testing.assert_allclose(P @ V, head_mean, rtol=1e-11, atol=1e-13)
