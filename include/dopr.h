@@ -166,6 +166,33 @@ DOPR_API dopr_status dopr_build_prefixes(dopr_model *model, dopr_store *store, i
                                          void *cuda_stream);
 
 /*
+ * Attention-based key token selection (Sec. 3.2.1), as the offline
+ * construction of Sec. 3.3 applies it: encode each document alone (its
+ * token ids at positions 0..n-1; no prefix, no score token), average the
+ * last layer's attention weights over the q heads into A[n][n] (row =
+ * attending token, causal), score token i by the mean of the top_p largest
+ * entries of column i (of its min(top_p, n - i) causal entries), keep the
+ * top_k most salient positions (equal salience to the lower position) and
+ * return them in ascending order with their final-layer states after the
+ * final RMSNorm -- the representations dopr_build_prefixes takes.  The paper
+ * leaves p open; top_p >= n gives the column mean.
+ *   doc_offsets [n_docs+1] int32, host: document d is doc_tokens[off[d] .. off[d+1]);
+ *               off[0] == 0, 1 <= n_d <= 2048 and n_d <= max_position.
+ *   doc_tokens  int32 token ids in [0, vocab), host.
+ *   1 <= top_k <= 256, top_p >= 1.
+ *   positions   [n_docs][top_k] int32, host: ascending, -1 past min(top_k, n_d).
+ *   x_out       [n_docs][top_k][hidden] bf16, host: the states at `positions`
+ *               (zero rows for -1).
+ *   salience    [off[n_docs]] float, host, or NULL: u of every token.
+ * Device memory of n^2 floats per document of a chunk is allocated for the
+ * call.  Synchronous.  Errors: INVALID_ARG, INCOMPLETE (model weights
+ * missing), OUT_OF_MEMORY, CUDA, TIMEOUT.
+ */
+DOPR_API dopr_status dopr_select_prefix_inputs(dopr_model *model, int32_t n_docs, const int32_t *doc_offsets,
+                                               const int32_t *doc_tokens, int32_t top_k, int32_t top_p,
+                                               int32_t *positions, void *x_out, float *salience, void *cuda_stream);
+
+/*
  * A stored layer of one document, read back for testing: k_out and v_out
  * (host, fp16 bits [m][n_kv_heads][head_dim], the dopr_store_put layout).
  * A document with m == 0 writes nothing.  Synchronous.

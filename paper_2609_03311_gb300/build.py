@@ -17,7 +17,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libdopr.so")
-SOURCES = ["abi.cu", "k_gemm.cu", "k_attn.cu", "k_attn_tc.cu", "k_rows.cu", "k_pack.cu", "k_pack_noalloc.cu"]
+SOURCES = ["abi.cu", "k_gemm.cu", "k_attn.cu", "k_attn_tc.cu", "k_select.cu", "k_rows.cu", "k_pack.cu", "k_pack_noalloc.cu"]
 HEADERS = [os.path.join(CSRC, "device_common.cuh"), os.path.join(CSRC, "internal.h"),
            os.path.join(ROOT, "include", "dopr.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

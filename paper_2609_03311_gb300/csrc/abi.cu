@@ -20,6 +20,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <memory>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -490,14 +491,29 @@ struct BuildArgs {
   const bf16* x;  // device, [total rows][hidden]
 };
 
+// Key token selection mode of run_layers: the packed tokens are documents'
+// token ids, each document one "pair" with no prefix and no score token; the
+// last layer runs in full, and after its QKV projection the selection kernels
+// rank the chunk's tokens, after its MLP the selected rows' final states are
+// gathered.
+struct SelectState {
+  int top_k, top_p;
+  float* A;        // device, the largest chunk's sum of n^2
+  int64_t* a_off;  // device, per chunk document
+  float* u;        // device, [all tokens]
+  int32_t* positions;
+  bf16* x;
+};
+
 dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cudaStream_t st,
-                       const BuildArgs* build = nullptr) {
+                       const BuildArgs* build = nullptr, SelectState* sel = nullptr) {
   Workspace& w = m->ws;
   const auto& c = m->cfg;
   const int H = c.hidden, F = c.ffn, L = c.n_layers, Hq = c.n_q_heads, Hkv = c.n_kv_heads;
   const int parts = H / GEMM_BN * GEMM_SS_PER_TILE;  // partial sums of squares per row from a residual epilogue
   const int mpad = ((s->max_m + 63) / 64) * 64;
   const int sms = m->num_sms;
+  const bool scoring = !build && !sel;
   auto gemm_cost = [](double M, double N, double K, double out_bytes) {
     return std::make_pair(2.0 * M * N * K, (M * K + N * K) * 2.0 + out_bytes);
   };
@@ -509,10 +525,10 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     double attn_keys = 0.0, prefix_rows = 0.0;
     for (int32_t sp = s0; sp < s1; ++sp) {
       const double Tp = w.h_tok_off[sp + 1] - w.h_tok_off[sp];
-      attn_keys += Tp * (build ? 0 : s->slot_m[w.h_sorted_slot[sp]]) + Tp * (Tp + 1) / 2;
+      attn_keys += Tp * (scoring ? s->slot_m[w.h_sorted_slot[sp]] : 0) + Tp * (Tp + 1) / 2;
     }
     for (int32_t it = plan.chunk_item[ci]; it < plan.chunk_item[ci + 1]; ++it) prefix_rows += w.h_items[it].m;
-    if (build) prefix_rows = 0.0;
+    if (!scoring) prefix_rows = 0.0;
     const double attn_flops = 4.0 * HEAD_DIM * Hq * attn_keys;
     const double attn_bytes = T * (2.0 * Hq + 2.0 * Hkv) * HEAD_DIM * 2 + prefix_rows * Hkv * 2 * HEAD_DIM * 2;
     // algorithmic bytes: operands once, outputs once (residual: read + write fp32, plus the next norm's bf16 operand)
@@ -532,7 +548,7 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     const int32_t np = s1 - s0;
     double last_keys = 0.0;  // keys seen by the score-token rows alone
     for (int32_t sp = s0; sp < s1; ++sp)
-      last_keys += s->slot_m[w.h_sorted_slot[sp]] + (w.h_tok_off[sp + 1] - w.h_tok_off[sp]);
+      last_keys += (scoring ? s->slot_m[w.h_sorted_slot[sp]] : 0) + (w.h_tok_off[sp + 1] - w.h_tok_off[sp]);
     const double attn_flops_last = 4.0 * HEAD_DIM * Hq * last_keys;
     const double attn_bytes_last = np * 2.0 * Hq * HEAD_DIM * 2 + T * 2.0 * Hkv * HEAD_DIM * 2 +
                                    prefix_rows * Hkv * 2 * HEAD_DIM * 2;
@@ -562,7 +578,8 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       // In the last layer only the score-token rows reach the score: after the full QKV
       // projection (every token's key and value is attended to), attention, O and the MLP
       // run on one compact row per pair.
-      const bool last = l + 1 == L;
+      const bool final_layer = l + 1 == L;
+      const bool last = scoring && final_layer;  // the scoring pass prunes its last layer to score rows
       GemmParams pq = base;  // QKV + attention-norm row scale + q/k norm + RoPE
       pq.N = m->qkv_dim;
       pq.K = H;
@@ -587,7 +604,36 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
           return launch_prefix_store(w.qkv, m->qkv_dim, Tc, t0, Hq, Hkv, w.tok_pair, w.tok_pos, w.sorted_slot,
                                      s->d_slot_row, s->d_slot_m, l, reinterpret_cast<f16*>(s->pool), st);
         }));
-        if (last) continue;
+        if (final_layer) continue;
+      }
+      if (sel && final_layer) {  // rank the chunk's tokens on this layer's q and k
+        SelectArgs sa{};
+        sa.qkv = w.qkv;
+        sa.ld_qkv = m->qkv_dim;
+        sa.Hq = Hq;
+        sa.Hkv = Hkv;
+        sa.tok_pair = w.tok_pair;
+        sa.tok_off = w.tok_off;
+        sa.t0 = t0;
+        sa.p0 = s0;
+        sa.n_docs = s1 - s0;
+        sa.n_rows = Tc;
+        sa.a_off = sel->a_off;
+        sa.A = sel->A;
+        sa.top_p = sel->top_p;
+        sa.top_k = sel->top_k;
+        sa.u = sel->u + t0;
+        sa.positions = sel->positions;
+        sa.x = sel->x;
+        std::vector<int64_t> aoff(s1 - s0);
+        int64_t acc = 0;
+        for (int32_t d = s0; d < s1; ++d) {
+          const int64_t nd = w.h_tok_off[d + 1] - w.h_tok_off[d];
+          aoff[d - s0] = acc;
+          acc += nd * nd;
+        }
+        CUDA_TRY(cudaMemcpyAsync(sel->a_off, aoff.data(), sizeof(int64_t) * aoff.size(), cudaMemcpyHostToDevice, st));
+        CUDA_TRY(launch_select(sa, st));
       }
       AttnArgs aa{};
       aa.items = w.items + (last ? plan.chunk_item[ci] : li0);
@@ -676,11 +722,21 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       CUDA_TRY(prof_launch(m, K_GEMM_DOWN, 1, last ? dn_last.first : dn.first, last ? dn_last.second : dn.second, st,
                            [&] { return launch_gemm(EPI_RESID_ADD, w.tm_act, m->tm_down[l], pd, sms, st); }));
     }
-    if (!build) {
+    if (scoring) {
       CUDA_TRY(prof_launch(m, K_SCORE, 1, 4.0 * H * (s1 - s0), (s1 - s0) * (H * 4.0 + 4.0), st, [&] {
         return launch_score(w.r_s, H, w.tok_off, t0, s0, s1, 1, w.perm, m->final_norm, m->score_head, c.rms_eps,
                             d_scores, st);
       }));
+    } else if (sel) {  // final states of the selected rows: the representations C_d
+      SelectArgs sa{};
+      sa.tok_off = w.tok_off;
+      sa.t0 = t0;
+      sa.p0 = s0;
+      sa.n_docs = s1 - s0;
+      sa.top_k = sel->top_k;
+      sa.positions = sel->positions;
+      sa.x = sel->x;
+      CUDA_TRY(launch_select_gather(sa, w.r, H, m->final_norm, c.rms_eps, st));
     }
   }
   return DOPR_OK;
@@ -794,7 +850,7 @@ dopr_status dopr_model_create(const dopr_model_config* cfg, dopr_model** out) {
   };
   cudaGetDevice(&m->device);
   cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
-  guard(gemm_setup() == cudaSuccess && attn_setup() == cudaSuccess && attn_tc_setup() == cudaSuccess
+  guard(gemm_setup() == cudaSuccess && attn_setup() == cudaSuccess && attn_tc_setup() == cudaSuccess && select_setup() == cudaSuccess
             ? DOPR_OK
             : fail(DOPR_ERR_CUDA, "kernel attribute setup failed: %s", cudaGetErrorString(cudaGetLastError())));
   if (st == DOPR_OK &&
@@ -1105,6 +1161,119 @@ dopr_status dopr_build_prefixes(dopr_model* m, dopr_store* s, int32_t n_docs, co
   for (int32_t d = 0; d < n_docs; ++d)
     for (int l = 0; l < L; ++l) STATUS_TRY(store_mark(s, slot[d], l, true));
   return DOPR_OK;
+}
+
+dopr_status dopr_select_prefix_inputs(dopr_model* m, int32_t n_docs, const int32_t* doc_offsets,
+                                      const int32_t* doc_tokens, int32_t top_k, int32_t top_p, int32_t* positions,
+                                      void* x_out, float* salience, void* cuda_stream) {
+  g_last_error.clear();
+  if (!m) return fail(DOPR_ERR_INVALID_ARG, "model is NULL");
+  const auto& c = m->cfg;
+  const int H = c.hidden, L = c.n_layers;
+  for (int k = 0; k < kind_count(); ++k)
+    for (int l = 0; l < (kind_is_global(k) ? 1 : L); ++l)
+      if (!m->have[k * L + l]) return fail(DOPR_ERR_INCOMPLETE, "weight kind %d layer %d was never put", k, l);
+  if (n_docs < 0) return fail(DOPR_ERR_INVALID_ARG, "n_docs < 0");
+  if (n_docs == 0) return DOPR_OK;
+  if (!doc_offsets || !doc_tokens || !positions || !x_out) return fail(DOPR_ERR_INVALID_ARG, "NULL array");
+  if (top_k < 1 || top_k > MAX_PREFIX) return fail(DOPR_ERR_INVALID_ARG, "top_k = %d outside [1, %d]", top_k, MAX_PREFIX);
+  if (top_p < 1) return fail(DOPR_ERR_INVALID_ARG, "top_p < 1");
+  if (doc_offsets[0] != 0) return fail(DOPR_ERR_INVALID_ARG, "doc_offsets[0] must be 0");
+  for (int32_t d = 0; d < n_docs; ++d) {
+    const int32_t nd = doc_offsets[d + 1] - doc_offsets[d];
+    if (nd < 1 || nd > SEL_MAX_N) return fail(DOPR_ERR_INVALID_ARG, "document %d: %d tokens outside [1, %d]", d, nd, SEL_MAX_N);
+    if (nd > c.max_position) return fail(DOPR_ERR_INVALID_ARG, "document %d: %d tokens beyond max_position", d, nd);
+  }
+  const int64_t T = doc_offsets[n_docs];
+  for (int64_t t = 0; t < T; ++t)
+    if (doc_tokens[t] < 0 || doc_tokens[t] >= c.vocab) return fail(DOPR_ERR_INVALID_ARG, "token %lld out of range", (long long)t);
+  CUDA_TRY(cudaSetDevice(m->device));
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  Workspace& w = m->ws;
+  // a store of one empty document gives the attention kernels a valid pool map
+  dopr_store* empty = nullptr;
+  STATUS_TRY(dopr_store_create(&c, 0, 256, &empty));
+  std::unique_ptr<dopr_store, void (*)(dopr_store*)> hold(empty, [](dopr_store* x) { dopr_store_destroy(x); });
+  dopr_status rs = ensure_call_buffers(m, n_docs, T, 0, 0);
+  if (rs != DOPR_OK) return rs;
+  std::vector<int32_t> tok_pos(T), tok_pair(T);
+  for (int32_t d = 0; d < n_docs; ++d) {
+    w.h_tok_off[d] = doc_offsets[d];
+    w.h_sorted_slot[d] = 0;
+    for (int32_t j = doc_offsets[d]; j < doc_offsets[d + 1]; ++j) {
+      tok_pos[j] = j - doc_offsets[d];
+      tok_pair[j] = d;
+    }
+  }
+  w.h_tok_off[n_docs] = (int32_t)T;
+  CUDA_TRY(cudaMemcpyAsync(w.tok_off, w.h_tok_off, sizeof(int32_t) * (n_docs + 1), cudaMemcpyHostToDevice, st));
+  CUDA_TRY(cudaMemcpyAsync(w.sorted_slot, w.h_sorted_slot, sizeof(int32_t) * n_docs, cudaMemcpyHostToDevice, st));
+  CUDA_TRY(cudaMemcpyAsync(w.tok_id, doc_tokens, sizeof(int32_t) * T, cudaMemcpyHostToDevice, st));
+  CUDA_TRY(cudaMemcpyAsync(w.tok_pos, tok_pos.data(), sizeof(int32_t) * T, cudaMemcpyHostToDevice, st));
+  CUDA_TRY(cudaMemcpyAsync(w.tok_pair, tok_pair.data(), sizeof(int32_t) * T, cudaMemcpyHostToDevice, st));
+  // chunks of whole documents; no prefix, so a chunk's documents form one attention run
+  const int TT = attn_tc_rows_per_head(c.n_q_heads / c.n_kv_heads);
+  Plan plan;
+  plan.n_tokens = T;
+  plan.chunk_pair.assign(1, 0);
+  plan.chunk_item.assign(1, 0);
+  plan.chunk_litem.assign(1, 0);
+  plan.chunk_tile.assign(1, 0);
+  std::vector<AttnTile> tiles;
+  std::vector<AttnItem> litems;
+  int64_t a_max = 0;
+  int32_t docs_max = 0;
+  for (int32_t s0 = 0; s0 < n_docs;) {
+    int32_t s1 = s0 + 1;
+    while (s1 < n_docs && w.h_tok_off[s1 + 1] - w.h_tok_off[s0] <= w.chunk_cap) ++s1;
+    plan_attention(w.h_tok_off, w.h_tok_off[s0], s0, s1, 0, 0, 0, TT, tiles, litems);
+    int64_t a = 0;
+    for (int32_t d = s0; d < s1; ++d) a += (int64_t)(doc_offsets[d + 1] - doc_offsets[d]) * (doc_offsets[d + 1] - doc_offsets[d]);
+    a_max = std::max(a_max, a);
+    docs_max = std::max(docs_max, s1 - s0);
+    plan.chunk_pair.push_back(s1);
+    plan.chunk_item.push_back(0);
+    plan.chunk_litem.push_back((int32_t)litems.size());
+    plan.chunk_tile.push_back((int32_t)tiles.size());
+    s0 = s1;
+  }
+  plan.n_litems = (int32_t)litems.size();
+  plan.n_tiles = (int32_t)tiles.size();
+  if (plan.n_litems > w.item_cap || plan.n_litems > w.h_item_cap || plan.n_tiles > w.tile_cap)
+    return fail(DOPR_ERR_UNSUPPORTED, "attention plan exceeds its buffers");
+  std::copy(litems.begin(), litems.end(), w.h_items);
+  std::copy(tiles.begin(), tiles.end(), w.h_tiles);
+  if (plan.n_litems > 0)
+    CUDA_TRY(cudaMemcpyAsync(w.items, w.h_items, sizeof(AttnItem) * plan.n_litems, cudaMemcpyHostToDevice, st));
+  if (plan.n_tiles > 0)
+    CUDA_TRY(cudaMemcpyAsync(w.tiles, w.h_tiles, sizeof(AttnTile) * plan.n_tiles, cudaMemcpyHostToDevice, st));
+  // selection buffers for this call
+  SelectState sel{top_k, top_p, nullptr, nullptr, nullptr, nullptr, nullptr};
+  auto cleanup = [&] {
+    dev_free(sel.A); dev_free(sel.a_off); dev_free(sel.u); dev_free(sel.positions); dev_free(sel.x);
+  };
+  if (dev_alloc(&sel.A, (size_t)a_max) != DOPR_OK || dev_alloc(&sel.a_off, (size_t)docs_max) != DOPR_OK ||
+      dev_alloc(&sel.u, (size_t)T) != DOPR_OK || dev_alloc(&sel.positions, (size_t)n_docs * top_k) != DOPR_OK ||
+      dev_alloc(&sel.x, (size_t)n_docs * top_k * H) != DOPR_OK) {
+    cleanup();
+    return fail(DOPR_ERR_OUT_OF_MEMORY, "selection buffers");
+  }
+  cudaError_t e = cudaMemsetAsync(w.err, 0, sizeof(int), st);
+  rs = e == cudaSuccess ? run_layers(m, empty, plan, nullptr, st, nullptr, &sel) : fail(DOPR_ERR_CUDA, "memset failed");
+  if (rs == DOPR_OK) {
+    e = cudaMemcpyAsync(positions, sel.positions, sizeof(int32_t) * n_docs * top_k, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(x_out, sel.x, sizeof(bf16) * (size_t)n_docs * top_k * H, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && salience) e = cudaMemcpyAsync(salience, sel.u, sizeof(float) * T, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(w.h_err, w.err, sizeof(int), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) rs = fail(DOPR_ERR_CUDA, "selection failed: %s", cudaGetErrorString(e));
+  } else {
+    cudaStreamSynchronize(st);
+  }
+  cleanup();
+  STATUS_TRY(rs);
+  return map_device_error(*w.h_err);
 }
 
 dopr_status dopr_debug_store_read(const dopr_store* s, int64_t doc_id, int32_t layer, void* k_out, void* v_out) {

@@ -288,6 +288,26 @@ cudaError_t launch_pack_tokens(const PackArgs& a, cudaStream_t st);
 void set_last_error_message(const std::string& msg);
 
 // Debug kernel: bounded wait on a barrier nothing completes.
+// Key token selection (k_select.cu), per chunk of whole documents (pairs p0 ..
+// p0 + n_docs - 1, chunk rows 0 .. n_rows - 1).
+constexpr int SEL_MAX_N = 2048;  // longest document the selection takes
+struct SelectArgs {
+  const f16* qkv;  // the chunk's q | k | v rows after the last layer's projection
+  int ld_qkv, Hq, Hkv;
+  const int32_t* tok_pair;  // packed token -> document (pair) index
+  const int32_t* tok_off;   // document -> first packed token
+  int t0, p0, n_docs, n_rows;
+  const int64_t* a_off;     // chunk document -> offset of its n x n A-bar in A
+  float* A;
+  int top_p, top_k;
+  float* u;                 // salience of chunk row t at u[t]
+  int32_t* positions;       // [all documents][top_k]
+  bf16* x;                  // [all documents][top_k][hidden]
+};
+cudaError_t select_setup();
+cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
+cudaError_t launch_select_gather(const SelectArgs& a, const float* r, int H, const bf16* gain, float eps,
+                                 cudaStream_t st);
 // Prefix build: K/V rows of chunk tokens [0, T) (packed tokens t0 + t) into the store pool.
 cudaError_t launch_prefix_store(const f16* qkv, int ld_qkv, int T, int t0, int Hq, int Hkv, const int32_t* tok_pair,
                                 const int32_t* tok_pos, const int32_t* pair_slot, const int64_t* slot_row,

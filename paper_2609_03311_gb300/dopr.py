@@ -75,6 +75,7 @@ def load():
         "dopr_profile_read": ([P, P, i32], i32),
         "dopr_build_prefixes": ([P, P, i32, P, P, P, i32, P], i32),
         "dopr_debug_store_read": ([P, i64, i32, P, P], i32),
+        "dopr_select_prefix_inputs": ([P, i32, P, P, i32, i32, P, P, P, P], i32),
         "dopr_last_error": ([], ctypes.c_char_p),
         "dopr_version": ([], ctypes.c_char_p),
     }
@@ -216,6 +217,22 @@ def build_prefixes(model: Model, store: Store, doc_ids, x_offsets, x: torch.Tens
                          (torch.cuda.current_stream().cuda_stream if x.is_cuda else 0))
     _check(load().dopr_build_prefixes(model._h, store._h, len(di), di.ctypes.data, xo.ctypes.data, _ptr(x),
                                       int(x.is_cuda), st))
+
+
+def select_prefix_inputs(model: Model, doc_offsets, doc_tokens, top_k: int, top_p: int, stream=None):
+    """Attention-based key token selection: (positions int32 [n_docs, top_k]
+    ascending with -1 padding, states bf16 [n_docs, top_k, hidden], salience
+    float32 [tokens])."""
+    off, tok = _host(doc_offsets, np.int32), _host(doc_tokens, np.int32)
+    n = len(off) - 1
+    H = model.cfg.hidden
+    pos = np.full((max(n, 1), top_k), -1, np.int32)
+    x = torch.zeros((max(n, 1), top_k, H), dtype=torch.bfloat16)
+    u = np.zeros(max(int(off[-1]) if n > 0 else 0, 1), np.float32)
+    st = ctypes.c_void_p(stream.cuda_stream if stream is not None else torch.cuda.current_stream().cuda_stream)
+    _check(load().dopr_select_prefix_inputs(model._h, n, off.ctypes.data, tok.ctypes.data, int(top_k), int(top_p),
+                                            pos.ctypes.data, _ptr(x), u.ctypes.data, st))
+    return pos[:n], x[:n], u[:int(off[-1]) if n > 0 else 0]
 
 
 def score(model: Model, store: Store, q_offsets, q_tokens, doc_ids, out=None, stream=None) -> torch.Tensor:
