@@ -362,60 +362,95 @@ struct Plan {
   std::vector<int32_t> chunk_item;   // and attention items [chunk_item[c], chunk_item[c+1]) (every pair)
   std::vector<int32_t> chunk_litem;  // mma.sync-kernel items [chunk_litem[c], chunk_litem[c+1])
   std::vector<int32_t> chunk_tile;   // tensor-core tiles [chunk_tile[c], chunk_tile[c+1])
-  int32_t n_items = 0, n_litems = 0, n_tiles = 0;
+  std::vector<int32_t> chunk_ltile;  // long tensor-core tiles, after all short ones
+  int32_t n_items = 0, n_litems = 0, n_tiles = 0, n_ltiles = 0;
 };
 
-// Cut the sorted pairs [pb, pe) of one document (chunk-relative token offsets
-// from `to`, t0 the chunk's first token) into tensor-core tiles of at most TT
-// tokens and ATTN_TC_MAX_KEYS key columns, and runs of pairs that do not fit
-// the key budget into mma.sync-kernel items.
-void plan_attention(const int32_t* to, int32_t t0, int32_t pb, int32_t pe, int32_t slot, int32_t m, int64_t pool_base,
-                    int TT, std::vector<AttnTile>& tiles, std::vector<AttnItem>& litems) {
-  auto c16 = [](int x) { return (x + 15) & ~15; };
-  auto fits = [&](int32_t p) { return TT > 0 && attn_tc_pair_fits(m, to[p + 1] - to[p]); };
-  const int pre64 = ((m + 63) / 64) * 64;
-  int32_t p = pb;
-  while (p < pe) {
-    int32_t q = p + 1;
-    if (!fits(p)) {
-      while (q < pe && q - p < ATTN_MAX_PAIRS && !fits(q)) ++q;
-      litems.push_back(AttnItem{p, q, slot, m});
-      p = q;
-      continue;
-    }
-    while (q < pe && fits(q)) ++q;
-    const int32_t end = to[q] - t0;
-    int32_t tok = to[p] - t0, pf = p;
-    while (tok < end) {
-      while (to[pf + 1] - t0 <= tok) ++pf;
-      int32_t n = 0, closed = 0, keys = 0, pp = pf;
-      while (n < TT && tok + n < end) {
-        const int32_t t = tok + n;
-        while (to[pp + 1] - t0 <= t) {  // pair pp lies wholly in the tile: its full segment
-          closed += c16(to[pp + 1] - to[pp]);
-          ++pp;
+// Attention plan of a call: tensor-core tiles of at most TT tokens -- short ones
+// within ATTN_TC_MAX_KEYS key columns, long ones (pairs whose own keys alone can
+// exceed that) without a key limit -- and, when G gives no tile shape, runs of
+// pairs for the mma.sync kernel.  Tiles keep at most ATTN_TC_MAX_SEGS pairs.
+struct AttnPlanner {
+  int TT = 0;
+  std::vector<AttnTile> tiles, ltiles;
+  std::vector<AttnItem> litems;
+
+  // The sorted pairs [pb, pe) of one document (token offsets `to`, t0 the chunk's first token).
+  void add(const int32_t* to, int32_t t0, int32_t pb, int32_t pe, int32_t slot, int32_t m, int64_t pool_base) {
+    auto c16 = [](int x) { return (x + 15) & ~15; };
+    auto fits = [&](int32_t p) { return attn_tc_pair_fits(m, to[p + 1] - to[p]); };
+    const int pre64 = ((m + 63) / 64) * 64;
+    int32_t p = pb;
+    while (p < pe) {
+      int32_t q = p + 1;
+      if (TT == 0) {
+        while (q < pe && q - p < ATTN_MAX_PAIRS) ++q;
+        litems.push_back(AttnItem{p, q, slot, m});
+        p = q;
+        continue;
+      }
+      const bool is_long = !fits(p);
+      while (q < pe && fits(q) != is_long) ++q;  // a run of pairs of one kind
+      std::vector<AttnTile>& out = is_long ? ltiles : tiles;
+      const int32_t end = to[q] - t0;
+      int32_t tok = to[p] - t0, pf = p;
+      while (tok < end) {
+        while (to[pf + 1] - t0 <= tok) ++pf;
+        int32_t n = 0, closed = 0, keys = 0, pp = pf;
+        while (n < TT && tok + n < end) {
+          const int32_t t = tok + n;
+          while (to[pp + 1] - t0 <= t) {  // pair pp lies wholly in the tile: its full segment
+            closed += c16(to[pp + 1] - to[pp]);
+            ++pp;
+          }
+          const int32_t k = pre64 + closed + c16(t - (to[pp] - t0) + 1);
+          if ((!is_long && k > ATTN_TC_MAX_KEYS) || pp - pf >= ATTN_TC_MAX_SEGS) break;
+          keys = k;
+          ++n;
         }
-        const int32_t k = pre64 + closed + c16(t - (to[pp] - t0) + 1);
-        if (k > ATTN_TC_MAX_KEYS) break;
-        keys = k;
-        ++n;
+        AttnTile tl{};
+        tl.pool_base = pool_base;
+        tl.tok_begin = tok;
+        tl.n_tok = n;
+        tl.m = m;
+        tl.n_keys = keys;
+        for (int32_t sp = pf; to[sp] - t0 < tok + n; ++sp) {
+          const int32_t ps = to[sp] - t0, nvis = std::min(to[sp + 1] - t0, tok + n) - ps;
+          tl.seg[tl.n_seg++] = (int32_t)(((uint32_t)nvis << 16) | (uint16_t)(int16_t)(ps - tok));
+        }
+        out.push_back(tl);
+        tok += n;
       }
-      AttnTile tl{};
-      tl.pool_base = pool_base;
-      tl.tok_begin = tok;
-      tl.n_tok = n;
-      tl.m = m;
-      tl.n_keys = keys;
-      for (int32_t sp = pf; to[sp] - t0 < tok + n; ++sp) {
-        const int32_t ps = to[sp] - t0, nvis = std::min(to[sp + 1] - t0, tok + n) - ps;
-        tl.seg[tl.n_seg++] = (int32_t)(((uint32_t)nvis << 16) | (uint16_t)(int16_t)(ps - tok));
-      }
-      tiles.push_back(tl);
-      tok += n;
+      p = q;
     }
-    p = q;
   }
-}
+  void close_chunk(Plan& plan) const {
+    plan.chunk_litem.push_back((int32_t)litems.size());
+    plan.chunk_tile.push_back((int32_t)tiles.size());
+    plan.chunk_ltile.push_back((int32_t)ltiles.size());
+  }
+  // Copy the plan to the workspace (host staging and device): the mma.sync items
+  // after the first n_items entries, the short tiles, then the long tiles.
+  dopr_status upload(Workspace& w, Plan& plan, int32_t n_items, cudaStream_t st) const {
+    plan.n_items = n_items;
+    plan.n_litems = (int32_t)litems.size();
+    plan.n_tiles = (int32_t)tiles.size();
+    plan.n_ltiles = (int32_t)ltiles.size();
+    if (n_items + plan.n_litems > w.item_cap || n_items + plan.n_litems > w.h_item_cap ||
+        plan.n_tiles + plan.n_ltiles > w.tile_cap)
+      return fail(DOPR_ERR_UNSUPPORTED, "attention plan exceeds its buffers");
+    std::copy(litems.begin(), litems.end(), w.h_items + n_items);
+    std::copy(tiles.begin(), tiles.end(), w.h_tiles);
+    std::copy(ltiles.begin(), ltiles.end(), w.h_tiles + tiles.size());
+    if (n_items + plan.n_litems > 0)
+      CUDA_TRY(cudaMemcpyAsync(w.items, w.h_items, sizeof(AttnItem) * (n_items + plan.n_litems),
+                               cudaMemcpyHostToDevice, st));
+    if (plan.n_tiles + plan.n_ltiles > 0)
+      CUDA_TRY(cudaMemcpyAsync(w.tiles, w.h_tiles, sizeof(AttnTile) * (plan.n_tiles + plan.n_ltiles),
+                               cudaMemcpyHostToDevice, st));
+    return DOPR_OK;
+  }
+};
 
 // Steps 1-4 of the engine.  Inputs are device pointers.  On return the packed
 // plan is on the device and the chunking in `plan`.
@@ -438,13 +473,13 @@ dopr_status run_packer(Model* m, Store* s, int32_t n, const int32_t* dqo, const 
   // chunks of whole pairs, then attention items (runs of one doc, <= ATTN_MAX_PAIRS),
   // and per chunk the tensor-core tiles and the mma.sync kernel's items
   const int cap = w.chunk_cap;
-  const int TT = attn_tc_rows_per_head(m->cfg.n_q_heads / m->cfg.n_kv_heads);
+  AttnPlanner ap;
+  ap.TT = attn_tc_rows_per_head(m->cfg.n_q_heads / m->cfg.n_kv_heads);
   plan.chunk_pair.assign(1, 0);
   plan.chunk_item.assign(1, 0);
   plan.chunk_litem.assign(1, 0);
   plan.chunk_tile.assign(1, 0);
-  std::vector<AttnTile> tiles;
-  std::vector<AttnItem> litems;
+  plan.chunk_ltile.assign(1, 0);
   int32_t items = 0;
   int32_t s0 = 0;
   while (s0 < n) {
@@ -459,28 +494,15 @@ dopr_status run_packer(Model* m, Store* s, int32_t n, const int32_t* dqo, const 
       const int32_t slot = w.h_sorted_slot[i], mm = s->slot_m[slot];
       for (int32_t a = i; a < j; a += ATTN_MAX_PAIRS)
         w.h_items[items++] = AttnItem{a, std::min(j, a + ATTN_MAX_PAIRS), slot, mm};
-      plan_attention(w.h_tok_off, w.h_tok_off[s0], i, j, slot, mm, s->slot_row[slot], TT, tiles, litems);
+      ap.add(w.h_tok_off, w.h_tok_off[s0], i, j, slot, mm, s->slot_row[slot]);
       i = j;
     }
     plan.chunk_pair.push_back(s1);
     plan.chunk_item.push_back(items);
-    plan.chunk_litem.push_back((int32_t)litems.size());
-    plan.chunk_tile.push_back((int32_t)tiles.size());
+    ap.close_chunk(plan);
     s0 = s1;
   }
-  plan.n_items = items;
-  plan.n_litems = (int32_t)litems.size();
-  plan.n_tiles = (int32_t)tiles.size();
-  if (items + plan.n_litems > w.item_cap || items + plan.n_litems > w.h_item_cap || plan.n_tiles > w.tile_cap)
-    return fail(DOPR_ERR_UNSUPPORTED, "attention plan exceeds its buffers");
-  std::copy(litems.begin(), litems.end(), w.h_items + items);
-  std::copy(tiles.begin(), tiles.end(), w.h_tiles);
-  if (items + plan.n_litems > 0)
-    CUDA_TRY(cudaMemcpyAsync(w.items, w.h_items, sizeof(AttnItem) * (items + plan.n_litems), cudaMemcpyHostToDevice,
-                             st));
-  if (plan.n_tiles > 0)
-    CUDA_TRY(cudaMemcpyAsync(w.tiles, w.h_tiles, sizeof(AttnTile) * plan.n_tiles, cudaMemcpyHostToDevice, st));
-  return DOPR_OK;
+  return ap.upload(w, plan, items, st);
 }
 
 // Prefix build mode of run_layers: the packed "tokens" are the selected document
@@ -557,7 +579,8 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     const int TT = attn_tc_rows_per_head(Hq / Hkv);
     CUtensorMap tm_q{}, tm_kv{};
     const int n_tiles = plan.chunk_tile[ci + 1] - plan.chunk_tile[ci];
-    if (n_tiles > 0 &&
+    const int n_ltiles = plan.chunk_ltile[ci + 1] - plan.chunk_ltile[ci];
+    if (n_tiles + n_ltiles > 0 &&
         !(make_tmap_16b_2d(&tm_q, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, TT, true, true) &&
           make_tmap_16b_2d(&tm_kv, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, 16, true, true)))
       return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for the QKV buffer");
@@ -569,6 +592,9 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     ta.Hq = Hq;
     ta.Hkv = Hkv;
     ta.err = w.err;
+    AttnTcArgs tl = ta;  // the long tiles, stored after every short tile
+    tl.tiles = w.tiles + plan.n_tiles + plan.chunk_ltile[ci];
+    tl.n_units = n_ltiles * Hkv;
     const int32_t li0 = plan.n_items + plan.chunk_litem[ci];
     const int32_t n_litems = plan.chunk_litem[ci + 1] - plan.chunk_litem[ci];
     const auto op_last = gemm_cost(np, H, m->o_dim, np * H * 10.0);
@@ -653,7 +679,8 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       aa.score_only = last ? 1 : 0;
       aa.pair_base = s0;
       aa.err = w.err;
-      const int attn_launches = (!last && ta.n_units > 0 ? 1 : 0) + (aa.n_items > 0 ? 1 : 0);
+      const int attn_launches = (!last && ta.n_units > 0 ? 1 : 0) + (!last && tl.n_units > 0 ? 1 : 0) +
+                                (aa.n_items > 0 ? 1 : 0);
       CUDA_TRY(prof_launch(m, K_ATTENTION, attn_launches, last ? attn_flops_last : attn_flops,
                            last ? attn_bytes_last : attn_bytes, st,
                            [&] {
@@ -663,6 +690,10 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
                              if (!last && ta.n_units > 0) {
                                ta.layer = l;
                                e = launch_attention_tc(tm_q, tm_kv, s->tm_pool, ta, sms, st);
+                             }
+                             if (e == cudaSuccess && !last && tl.n_units > 0) {
+                               tl.layer = l;
+                               e = launch_attention_tc_long(tm_q, tm_kv, s->tm_pool, tl, sms, st);
                              }
                              if (e == cudaSuccess && aa.n_items > 0) e = launch_attention(s->tm_pool, aa, st);
                              return e;
@@ -1107,35 +1138,25 @@ dopr_status dopr_build_prefixes(dopr_model* m, dopr_store* s, int32_t n_docs, co
     CUDA_TRY(cudaMemcpyAsync(w.tok_pos, tok_pos.data(), sizeof(int32_t) * T, cudaMemcpyHostToDevice, st));
     CUDA_TRY(cudaMemcpyAsync(w.tok_pair, tok_pair.data(), sizeof(int32_t) * T, cudaMemcpyHostToDevice, st));
     // chunks of whole documents; attention with no prefix, so a chunk's documents form one run
-    const int TT = attn_tc_rows_per_head(c.n_q_heads / c.n_kv_heads);
+    AttnPlanner ap;
+    ap.TT = attn_tc_rows_per_head(c.n_q_heads / c.n_kv_heads);
     Plan plan;
     plan.n_tokens = T;
     plan.chunk_pair.assign(1, 0);
     plan.chunk_item.assign(1, 0);
     plan.chunk_litem.assign(1, 0);
     plan.chunk_tile.assign(1, 0);
-    std::vector<AttnTile> tiles;
-    std::vector<AttnItem> litems;
+    plan.chunk_ltile.assign(1, 0);
     for (int32_t s0 = 0; s0 < n;) {
       int32_t s1 = s0 + 1;
       while (s1 < n && w.h_tok_off[s1 + 1] - w.h_tok_off[s0] <= w.chunk_cap) ++s1;
-      plan_attention(w.h_tok_off, w.h_tok_off[s0], s0, s1, 0, 0, 0, TT, tiles, litems);
+      ap.add(w.h_tok_off, w.h_tok_off[s0], s0, s1, 0, 0, 0);
       plan.chunk_pair.push_back(s1);
       plan.chunk_item.push_back(0);
-      plan.chunk_litem.push_back((int32_t)litems.size());
-      plan.chunk_tile.push_back((int32_t)tiles.size());
+      ap.close_chunk(plan);
       s0 = s1;
     }
-    plan.n_litems = (int32_t)litems.size();
-    plan.n_tiles = (int32_t)tiles.size();
-    if (plan.n_litems > w.item_cap || plan.n_litems > w.h_item_cap || plan.n_tiles > w.tile_cap)
-      return fail(DOPR_ERR_UNSUPPORTED, "attention plan exceeds its buffers");
-    std::copy(litems.begin(), litems.end(), w.h_items);
-    std::copy(tiles.begin(), tiles.end(), w.h_tiles);
-    if (plan.n_litems > 0)
-      CUDA_TRY(cudaMemcpyAsync(w.items, w.h_items, sizeof(AttnItem) * plan.n_litems, cudaMemcpyHostToDevice, st));
-    if (plan.n_tiles > 0)
-      CUDA_TRY(cudaMemcpyAsync(w.tiles, w.h_tiles, sizeof(AttnTile) * plan.n_tiles, cudaMemcpyHostToDevice, st));
+    STATUS_TRY(ap.upload(w, plan, 0, st));
     // the representations on the device
     const bf16* dx = static_cast<const bf16*>(x);
     bf16* stage = nullptr;
@@ -1212,41 +1233,31 @@ dopr_status dopr_select_prefix_inputs(dopr_model* m, int32_t n_docs, const int32
   CUDA_TRY(cudaMemcpyAsync(w.tok_pos, tok_pos.data(), sizeof(int32_t) * T, cudaMemcpyHostToDevice, st));
   CUDA_TRY(cudaMemcpyAsync(w.tok_pair, tok_pair.data(), sizeof(int32_t) * T, cudaMemcpyHostToDevice, st));
   // chunks of whole documents; no prefix, so a chunk's documents form one attention run
-  const int TT = attn_tc_rows_per_head(c.n_q_heads / c.n_kv_heads);
+  AttnPlanner ap;
+  ap.TT = attn_tc_rows_per_head(c.n_q_heads / c.n_kv_heads);
   Plan plan;
   plan.n_tokens = T;
   plan.chunk_pair.assign(1, 0);
   plan.chunk_item.assign(1, 0);
   plan.chunk_litem.assign(1, 0);
   plan.chunk_tile.assign(1, 0);
-  std::vector<AttnTile> tiles;
-  std::vector<AttnItem> litems;
+  plan.chunk_ltile.assign(1, 0);
   int64_t a_max = 0;
   int32_t docs_max = 0;
   for (int32_t s0 = 0; s0 < n_docs;) {
     int32_t s1 = s0 + 1;
     while (s1 < n_docs && w.h_tok_off[s1 + 1] - w.h_tok_off[s0] <= w.chunk_cap) ++s1;
-    plan_attention(w.h_tok_off, w.h_tok_off[s0], s0, s1, 0, 0, 0, TT, tiles, litems);
+    ap.add(w.h_tok_off, w.h_tok_off[s0], s0, s1, 0, 0, 0);
     int64_t a = 0;
     for (int32_t d = s0; d < s1; ++d) a += (int64_t)(doc_offsets[d + 1] - doc_offsets[d]) * (doc_offsets[d + 1] - doc_offsets[d]);
     a_max = std::max(a_max, a);
     docs_max = std::max(docs_max, s1 - s0);
     plan.chunk_pair.push_back(s1);
     plan.chunk_item.push_back(0);
-    plan.chunk_litem.push_back((int32_t)litems.size());
-    plan.chunk_tile.push_back((int32_t)tiles.size());
+    ap.close_chunk(plan);
     s0 = s1;
   }
-  plan.n_litems = (int32_t)litems.size();
-  plan.n_tiles = (int32_t)tiles.size();
-  if (plan.n_litems > w.item_cap || plan.n_litems > w.h_item_cap || plan.n_tiles > w.tile_cap)
-    return fail(DOPR_ERR_UNSUPPORTED, "attention plan exceeds its buffers");
-  std::copy(litems.begin(), litems.end(), w.h_items);
-  std::copy(tiles.begin(), tiles.end(), w.h_tiles);
-  if (plan.n_litems > 0)
-    CUDA_TRY(cudaMemcpyAsync(w.items, w.h_items, sizeof(AttnItem) * plan.n_litems, cudaMemcpyHostToDevice, st));
-  if (plan.n_tiles > 0)
-    CUDA_TRY(cudaMemcpyAsync(w.tiles, w.h_tiles, sizeof(AttnTile) * plan.n_tiles, cudaMemcpyHostToDevice, st));
+  STATUS_TRY(ap.upload(w, plan, 0, st));
   // selection buffers for this call
   SelectState sel{top_k, top_p, nullptr, nullptr, nullptr, nullptr, nullptr};
   auto cleanup = [&] {

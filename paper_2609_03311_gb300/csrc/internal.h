@@ -256,6 +256,9 @@ cudaError_t attn_tc_setup();
 // buffer, box 64 x 16; tm_pool: the store pool, box 64 x 64 (all fp16, 128-byte swizzle).
 cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool,
                                 const AttnTcArgs& a, int num_sms, cudaStream_t st);
+// Tiles with more than ATTN_TC_MAX_KEYS key columns (same maps and arguments).
+cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool,
+                                     const AttnTcArgs& a, int num_sms, cudaStream_t st);
 
 // Packer.
 struct PackArgs {

@@ -540,10 +540,389 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
+// ============================================================================
+// Long tiles: more key columns than one TMEM region holds (long queries, the
+// longest prefixes with long queries, uncompressed documents).  One unit at a
+// time per CTA, one softmax warpgroup, the keys in 128-column chunks through
+// two S buffers: pass A computes S chunk by chunk for the exact row maximum,
+// pass B computes each chunk again, writes P and accumulates O = P V in its own
+// 128 TMEM columns.  The row results are the short kernel's: the same maximum,
+// the same 16-key sums in key order, the same MMA steps.
+namespace lt {
+constexpr int Q_STAGES = 2, K_STAGES = 3, V_STAGES = 3, P_STAGES = 2;
+constexpr int CH = 128;  // key columns per S chunk
+constexpr int THREADS = 64 + 128;
+constexpr uint32_t O_COL = 0, S_COL = 128;  // S buffer b at S_COL + CH * b
+constexpr int OFF_Q = 0;
+constexpr int OFF_K = OFF_Q + Q_STAGES * Q_BYTES;
+constexpr int OFF_V = OFF_K + K_STAGES * KV_BYTES;
+constexpr int OFF_P = OFF_V + V_STAGES * KV_BYTES;
+constexpr int OFF_BAR = OFF_P + P_STAGES * P_BYTES;
+constexpr int B_Q_FULL = 0, B_Q_EMPTY = B_Q_FULL + Q_STAGES;
+constexpr int B_K_FULL = B_Q_EMPTY + Q_STAGES, B_K_EMPTY = B_K_FULL + K_STAGES;
+constexpr int B_V_FULL = B_K_EMPTY + K_STAGES, B_V_EMPTY = B_V_FULL + V_STAGES;
+constexpr int B_P_FULL = B_V_EMPTY + V_STAGES, B_P_EMPTY = B_P_FULL + P_STAGES;
+constexpr int B_S_FULL = B_P_EMPTY + P_STAGES, B_S_FREE = B_S_FULL + 2;
+constexpr int B_O_FULL = B_S_FREE + 2, B_O_FREE = B_O_FULL + 1, B_DRAIN = B_O_FREE + 1, N_BARS = B_DRAIN + 1;
+constexpr int SMEM_BYTES = 1024 + OFF_BAR + N_BARS * 8 + 16;
+static_assert(SMEM_BYTES <= 227 * 1024, "shared memory budget");
+static_assert(B_V_FULL + V_STAGES <= 32, "producer arm mask");
+}  // namespace lt
+
+__global__ void __launch_bounds__(lt::THREADS, 1)
+    k_attn_tc_long(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
+                   const __grid_constant__ CUtensorMap tm_pool, AttnTcArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t s0 = smem_u32(smem);
+  const uint32_t sQ = s0 + lt::OFF_Q, sK = s0 + lt::OFF_K, sV = s0 + lt::OFF_V, sP = s0 + lt::OFF_P;
+  auto bar = [&](int i) { return s0 + lt::OFF_BAR + 8u * static_cast<uint32_t>(i); };
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + lt::OFF_BAR + lt::N_BARS * 8);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = a.Hq / a.Hkv;
+  const int TT = TILE_M / G;
+  const int n_local = blockIdx.x < a.n_units ? (a.n_units - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
+  auto unit_of = [&](int i) { return blockIdx.x + i * gridDim.x; };
+  auto blocks_of = [](int n_keys) { return (n_keys + KBLK - 1) / KBLK; };
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < lt::Q_STAGES; ++i) {
+      mbar_init(bar(lt::B_Q_FULL + i), 1);
+      mbar_init(bar(lt::B_Q_EMPTY + i), 1);
+    }
+    for (int i = 0; i < lt::K_STAGES; ++i) {
+      mbar_init(bar(lt::B_K_FULL + i), 1);
+      mbar_init(bar(lt::B_K_EMPTY + i), 1);
+    }
+    for (int i = 0; i < lt::V_STAGES; ++i) {
+      mbar_init(bar(lt::B_V_FULL + i), 1);
+      mbar_init(bar(lt::B_V_EMPTY + i), 1);
+    }
+    for (int i = 0; i < lt::P_STAGES; ++i) {
+      mbar_init(bar(lt::B_P_FULL + i), 4);
+      mbar_init(bar(lt::B_P_EMPTY + i), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(bar(lt::B_S_FULL + i), 1);
+      mbar_init(bar(lt::B_S_FREE + i), 4);
+    }
+    mbar_init(bar(lt::B_O_FULL), 1);
+    mbar_init(bar(lt::B_O_FREE), 4);
+    mbar_init(bar(lt::B_DRAIN), 1);
+    fence_mbar_init();
+    tma_prefetch_desc(&tm_q);
+    tma_prefetch_desc(&tm_kv);
+    tma_prefetch_desc(&tm_pool);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ======================= TMA producer: Q; pass A's K blocks; pass B's K and V blocks chunk by chunk
+      Ring rq, rk, rv;
+      uint32_t armed = 0, armed_par = 0;
+      auto arm = [&](int b, uint32_t par, uint32_t bytes) {
+        mbar_arrive_expect_tx(bar(b), bytes);
+        armed |= 1u << b;
+        armed_par = (armed_par & ~(1u << b)) | (par << b);
+      };
+      // a block stream of one tile's K or V rows: blocks must be issued in order 0, 1, ...
+      struct Stream {
+        int kv, si, k, sv, pool_row, col0;
+      };
+      auto start = [&](const AttnTile* tp, int g, int kv) {
+        Stream st;
+        st.kv = kv;
+        st.si = 0;
+        st.k = 0;
+        st.sv = tp->seg[0];
+        st.pool_row = static_cast<int>(tp->pool_base + ((static_cast<int64_t>(a.layer) * 2 + kv) * a.Hkv + g) * tp->m);
+        st.col0 = (a.Hq + kv * a.Hkv + g) * HEAD_DIM;
+        return st;
+      };
+      auto issue_block = [&](const AttnTile* tp, Stream& st, int j) -> bool {
+        Ring& r = st.kv ? rv : rk;
+        const int stages = st.kv ? lt::V_STAGES : lt::K_STAGES;
+        const int full0 = st.kv ? lt::B_V_FULL : lt::B_K_FULL, empty0 = st.kv ? lt::B_V_EMPTY : lt::B_K_EMPTY;
+        if (!mbar_wait(bar(empty0 + r.stage), r.phase ^ 1u, a.err, WAIT_TIMEOUT_NS)) return false;
+        const uint32_t dst = (st.kv ? sV : sK) + r.stage * KV_BYTES;
+        const uint32_t fb = bar(full0 + r.stage);
+        if (j * KBLK < ceil64(tp->m)) {
+          arm(full0 + r.stage, r.phase, KV_BYTES);
+          for (int h = 0; h < 2; ++h) tma_load_2d(dst + h * KV_HALF, &tm_pool, fb, h * 64, st.pool_row + j * KBLK);
+        } else {
+          const int groups = min(KBLK, tp->n_keys - j * KBLK) / GROUP_ROWS;
+          arm(full0 + r.stage, r.phase, groups * GROUP_BYTES);
+          for (int q = 0; q < groups; ++q) {
+            for (int h = 0; h < 2; ++h)
+              tma_load_2d(dst + q * GROUP_ROWS * 128 + h * KV_HALF, &tm_kv, fb, st.col0 + h * 64,
+                          tp->tok_begin + seg_start(st.sv) + st.k);
+            st.k += GROUP_ROWS;
+            if (st.k >= seg_len(st.sv) && st.si + 1 < ATTN_TC_MAX_SEGS) {
+              st.k = 0;
+              st.sv = tp->seg[++st.si];
+            }
+          }
+        }
+        r.next(stages);
+        return true;
+      };
+      bool ok = true;
+      for (int i = 0; i < n_local && ok; ++i) {
+        const int u = unit_of(i);
+        const AttnTile* tp = a.tiles + u / a.Hkv;
+        const int g = u % a.Hkv;
+        const int nb = blocks_of(tp->n_keys);
+        if (i + 1 < n_local) prefetch_tile(a.tiles + unit_of(i + 1) / a.Hkv);
+        if (!mbar_wait(bar(lt::B_Q_EMPTY + rq.stage), rq.phase ^ 1u, a.err, WAIT_TIMEOUT_NS)) {
+          ok = false;
+          break;
+        }
+        arm(lt::B_Q_FULL + rq.stage, rq.phase, Q_BYTES);
+        for (int hh = 0; hh < G; ++hh)
+          for (int h = 0; h < 2; ++h)
+            tma_load_2d(sQ + rq.stage * Q_BYTES + h * Q_HALF + hh * TT * 128, &tm_q, bar(lt::B_Q_FULL + rq.stage),
+                        (g * G + hh) * HEAD_DIM + h * 64, tp->tok_begin);
+        rq.next(lt::Q_STAGES);
+        Stream ka = start(tp, g, 0);
+        for (int j = 0; j < nb && ok; ++j) ok = issue_block(tp, ka, j);
+        Stream kb = start(tp, g, 0), vb = start(tp, g, 1);
+        for (int c = 0; c * 2 < nb && ok; ++c) {
+          for (int j = 2 * c; j < min(nb, 2 * c + 2) && ok; ++j) ok = issue_block(tp, kb, j);
+          for (int j = 2 * c; j < min(nb, 2 * c + 2) && ok; ++j) ok = issue_block(tp, vb, j);
+        }
+      }
+      if (!ok) {
+        for (int b = 0; b < 32; ++b)
+          if (armed & (1u << b)) mbar_wait(bar(b), (armed_par >> b) & 1u, a.err, 100000000ull);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ======================= MMA issuer
+      Ring rq, rk, rv, rp;
+      uint32_t cc = 0;  // S chunks issued (both passes, all units): buffer cc & 1
+      bool ok = true;
+      auto wait = [&](int b, uint32_t par) { return ok = ok && mbar_wait(bar(b), par, a.err, WAIT_TIMEOUT_NS); };
+      // S of key chunk c (its one or two 64-key blocks from the K ring) into buffer cc & 1
+      auto issue_s = [&](int c, int nb) -> bool {
+        const uint32_t buf = cc & 1u;
+        if (!wait(lt::B_S_FREE + buf, ((cc >> 1) & 1u) ^ 1u)) return false;
+        tc_fence_after();
+        const uint64_t qd = umma_desc_sw128(sQ + rq.stage * Q_BYTES);
+        for (int j = 2 * c; j < min(nb, 2 * c + 2); ++j) {
+          if (!wait(lt::B_K_FULL + rk.stage, rk.phase)) return false;
+          tc_fence_after();
+          const uint64_t kd = umma_desc_sw128(sK + rk.stage * KV_BYTES);
+#pragma unroll
+          for (int ks = 0; ks < HEAD_DIM / 16; ++ks)
+            umma_f16(tmem + lt::S_COL + lt::CH * buf + (j - 2 * c) * KBLK, qd + ((ks >> 2) * Q_HALF + (ks & 3) * 32) / 16,
+                     kd + ((ks >> 2) * KV_HALF + (ks & 3) * 32) / 16, IDESC_S, ks > 0);
+          umma_commit(bar(lt::B_K_EMPTY + rk.stage));
+          rk.next(lt::K_STAGES);
+        }
+        umma_commit(bar(lt::B_S_FULL + buf));
+        ++cc;
+        return true;
+      };
+      for (int i = 0; i < n_local && ok; ++i) {
+        const int n_keys = a.tiles[unit_of(i) / a.Hkv].n_keys;
+        const int nb = blocks_of(n_keys), nc = (nb + 1) / 2;
+        if (!wait(lt::B_Q_FULL + rq.stage, rq.phase)) break;
+        tc_fence_after();
+        for (int c = 0; c < nc && ok; ++c) issue_s(c, nb);  // pass A
+        if (ok) issue_s(0, nb);                              // pass B
+        for (int c = 0; c < nc && ok; ++c) {
+          if (c + 1 < nc && !issue_s(c + 1, nb)) break;
+          if (c == 0 && !wait(lt::B_O_FREE, (static_cast<uint32_t>(i) & 1u) ^ 1u)) break;
+          for (int j = 2 * c; j < min(nb, 2 * c + 2) && ok; ++j) {
+            if (!wait(lt::B_P_FULL + rp.stage, rp.phase) || !wait(lt::B_V_FULL + rv.stage, rv.phase)) break;
+            tc_fence_after();
+            const int steps = min(KBLK, n_keys - j * KBLK) / 16;
+            const uint64_t pd = umma_desc_sw128(sP + rp.stage * P_BYTES);
+            const uint64_t vd = umma_desc_sw128_mn(sV + rv.stage * KV_BYTES, KV_HALF, 1024);
+            for (int kk = 0; kk < steps; ++kk)
+              umma_f16(tmem + lt::O_COL, pd + (kk * 32) / 16, vd + (kk * 2048) / 16, IDESC_O, (j | kk) != 0);
+            umma_commit(bar(lt::B_P_EMPTY + rp.stage));
+            umma_commit(bar(lt::B_V_EMPTY + rv.stage));
+            rp.next(lt::P_STAGES);
+            rv.next(lt::V_STAGES);
+          }
+        }
+        if (!ok) break;
+        umma_commit(bar(lt::B_O_FULL));
+        umma_commit(bar(lt::B_Q_EMPTY + rq.stage));
+        rq.next(lt::Q_STAGES);
+      }
+      umma_commit(bar(lt::B_DRAIN));
+      mbar_wait(bar(lt::B_DRAIN), 0, a.err, ok ? WAIT_TIMEOUT_NS : 100000000ull);
+    }
+  } else {
+    // ======================= softmax + epilogue: warps 2..5 -> TMEM lane quarters 2, 3, 0, 1
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;
+    const int jj = r % TT;  // this row's token within the tile (its q head is r / TT)
+    const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(HEAD_DIM));
+    uint8_t* prow0 = smem + lt::OFF_P + r * 128;
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    Ring rp;
+    uint32_t cc = 0;
+    bool ok = true;
+    for (int i = 0; i < n_local && ok; ++i) {
+      const int u = unit_of(i);
+      if (i + 1 < n_local) prefetch_tile(a.tiles + unit_of(i + 1) / a.Hkv);
+      const AttnTile* tp = a.tiles + u / a.Hkv;
+      const int g = u % a.Hkv;
+      const int m = tp->m, n_tok = tp->n_tok, n_seg = tp->n_seg;
+      const int pre64 = ceil64(m);
+      const int nb = blocks_of(tp->n_keys), nc = (nb + 1) / 2, ncol = nb * KBLK;
+      const bool valid = jj < n_tok;
+      int olo = INT_MAX, ohi = -1;
+      if (valid) {
+        int seg = pre64;
+        for (int si = 0; si < n_seg; ++si) {
+          const int sv = tp->seg[si];
+          const int st = seg_start(sv), len = seg_len(sv);
+          if (jj < st + len) {
+            olo = seg;
+            ohi = seg + (jj - st);
+            break;
+          }
+          seg += ceil16(len);
+        }
+      }
+      const int wlo = __reduce_min_sync(0xffffffffu, olo);
+      const int whi = __reduce_max_sync(0xffffffffu, ohi);
+      auto chunk_live = [&](int c0) { return c0 < m || (c0 <= whi && c0 + 31 >= wlo); };
+      auto vis_mask = [&](int c0) { return bits_in(-c0, m - c0) | bits_in(olo - c0, ohi + 1 - c0); };
+      // ---- pass A: the row maximum, chunk by chunk
+      float mx = -INFINITY;
+      for (int c = 0; c < nc && ok; ++c) {
+        const uint32_t buf = cc & 1u;
+        if (!mbar_wait(bar(lt::B_S_FULL + buf), (cc >> 1) & 1u, a.err, WAIT_TIMEOUT_NS)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        for (int c0 = c * lt::CH; c0 < min(ncol, c * lt::CH + lt::CH); c0 += 32) {
+          if (!chunk_live(c0)) continue;
+          uint32_t v[32];
+          tmem_ld32(lane_base + lt::S_COL + lt::CH * buf + (c0 - c * lt::CH), v);
+          tmem_ld_wait();
+          mx = fmaxf(mx, masked_max32(v, vis_mask(c0)));
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(lt::B_S_FREE + buf));
+        ++cc;
+      }
+      if (!ok) break;
+      const float mxs = (mx == -INFINITY) ? 0.f : mx * scale_log2;
+      // ---- pass B: P per 64-key block, 16-key sums in key order
+      float sum = 0.f;
+      for (int c = 0; c < nc && ok; ++c) {
+        const uint32_t buf = cc & 1u;
+        if (!mbar_wait(bar(lt::B_S_FULL + buf), (cc >> 1) & 1u, a.err, WAIT_TIMEOUT_NS)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        for (int j = 2 * c; j < min(nb, 2 * c + 2); ++j) {
+          if (!mbar_wait(bar(lt::B_P_EMPTY + rp.stage), rp.phase ^ 1u, a.err, WAIT_TIMEOUT_NS)) {
+            ok = false;
+            break;
+          }
+          uint8_t* prow = prow0 + rp.stage * P_BYTES;
+#pragma unroll
+          for (int hf = 0; hf < 2; ++hf) {
+            const int cb = j * KBLK + 32 * hf;
+            if (chunk_live(cb)) {
+              uint32_t v[32];
+              tmem_ld32(lane_base + lt::S_COL + lt::CH * buf + (cb - c * lt::CH), v);
+              tmem_ld_wait();
+              sum = exp_chunk(v, vis_mask(cb), scale_log2, mxs, sum, prow, hf, r);
+            } else {
+              zero_chunk(prow, hf, r);
+            }
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar(lt::B_P_FULL + rp.stage));
+          rp.next(lt::P_STAGES);
+        }
+        if (!ok) break;
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(lt::B_S_FREE + buf));
+        ++cc;
+      }
+      if (!ok) break;
+      // ---- epilogue: O / sum -> fp16, staged through this warp's own P lines
+      if (!mbar_wait(bar(lt::B_O_FULL), static_cast<uint32_t>(i) & 1u, a.err, WAIT_TIMEOUT_NS)) break;
+      tc_fence_after();
+      const float inv = sum > 0.f ? 1.f / sum : 0.f;
+      uint8_t* stg = smem + lt::OFF_P + quarter * 32 * 128;
+      auto stg_row = [&](int rr) { return stg + (rr >> 4) * P_BYTES + (rr & 15) * 256; };
+#pragma unroll 1
+      for (int c0 = 0; c0 < HEAD_DIM; c0 += 32) {
+        uint32_t v[32];
+        tmem_ld32(lane_base + lt::O_COL + c0, v);
+        tmem_ld_wait();
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const uint32_t* x = v + 8 * q;
+          uint4 o;
+          o.x = pack_f16x2(__uint_as_float(x[0]) * inv, __uint_as_float(x[1]) * inv);
+          o.y = pack_f16x2(__uint_as_float(x[2]) * inv, __uint_as_float(x[3]) * inv);
+          o.z = pack_f16x2(__uint_as_float(x[4]) * inv, __uint_as_float(x[5]) * inv);
+          o.w = pack_f16x2(__uint_as_float(x[6]) * inv, __uint_as_float(x[7]) * inv);
+          *reinterpret_cast<uint4*>(stg_row(lane) + (((c0 / 8 + q) ^ (lane & 7)) << 4)) = o;
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(lt::B_O_FREE));
+      {
+        const int half = lane >> 4, ch = lane & 15;
+#pragma unroll 4
+        for (int it = 0; it < 16; ++it) {
+          const int rr = 2 * it + half;
+          const int row = quarter * 32 + rr;
+          const int j2 = row % TT;
+          if (j2 < n_tok) {
+            const uint4 x = *reinterpret_cast<const uint4*>(stg_row(rr) + ((ch ^ (rr & 7)) << 4));
+            *reinterpret_cast<uint4*>(a.out + static_cast<int64_t>(tp->tok_begin + j2) * a.ld_out +
+                                      (g * G + row / TT) * HEAD_DIM + ch * 8) = x;
+          }
+        }
+      }
+      __syncwarp();
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
 }  // namespace
 
 cudaError_t attn_tc_setup() {
-  return cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  const cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(k_attn_tc_long, cudaFuncAttributeMaxDynamicSharedMemorySize, lt::SMEM_BYTES);
 }
 
 cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool,
@@ -551,6 +930,14 @@ cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_k
   if (a.n_units <= 0) return cudaSuccess;
   const int grid = a.n_units < num_sms ? a.n_units : num_sms;
   k_attn_tc<<<grid, THREADS, SMEM_BYTES, st>>>(tm_q, tm_kv, tm_pool, a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool,
+                                     const AttnTcArgs& a, int num_sms, cudaStream_t st) {
+  if (a.n_units <= 0) return cudaSuccess;
+  const int grid = a.n_units < num_sms ? a.n_units : num_sms;
+  k_attn_tc_long<<<grid, lt::THREADS, lt::SMEM_BYTES, st>>>(tm_q, tm_kv, tm_pool, a);
   return cudaGetLastError();
 }
 
