@@ -76,6 +76,8 @@ def load(lib_path: str | None = None):
     lib.oracle_attn_probs.argtypes = [P, P, ctypes.c_int, ctypes.c_int, f64, P]
     lib.oracle_salience.argtypes = [ctypes.c_int, P, ctypes.c_int, P]
     lib.oracle_select_topk.argtypes = [ctypes.c_int, P, ctypes.c_int, P]
+    lib.oracle_mlp_head.argtypes = [P, P, ctypes.c_int, P, P, P, f64, ctypes.c_int]
+    lib.oracle_mlp_head.restype = f64
     lib.oracle_score_head.argtypes = [P, P]
     lib.oracle_score_head.restype = f64
     lib.oracle_embed.argtypes = [P, ctypes.c_int, P, P]
@@ -228,6 +230,14 @@ class OracleModel:
     def score_head(self, h) -> float:
         h = _f64(h)
         return float(self.lib.oracle_score_head(self.ref, _ptr(h)))
+
+    def mlp_head(self, h, head: dict) -> float:
+        """The MLP scoring head on a final state h [H]; head: w1 bf16 [d, H],
+        b1 bf16 [d], w2 bf16 [d], b2 float, act int."""
+        h = _f64(h)
+        w1, b1, w2 = _u16(head["w1"]), _u16(head["b1"]), _u16(head["w2"])
+        return float(self.lib.oracle_mlp_head(self.ref, _ptr(h), int(w1.shape[0]), _ptr(w1), _ptr(b1), _ptr(w2),
+                                              float(head["b2"]), int(head["act"])))
 
     def score_pairs(self, q_offsets, q_tokens, pair_doc, docs) -> np.ndarray:
         """docs: list of (K, V) per document index, each [L,m,Hkv,D] (fp64

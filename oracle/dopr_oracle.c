@@ -27,7 +27,8 @@
  *     frequency theta^(-2i/D);
  *   - q head h reads kv head floor(h / G), G = Hq / Hkv;
  *   - RMSNorm(x) = x / sqrt(mean(x^2) + eps) * g;
- *   - score = <W_s[0], RMSNorm(h_last) * g_final> - <W_s[1], ...>.
+ *   - score = <W_s[0], RMSNorm(h_last) * g_final> - <W_s[1], ...> (or, with the
+ *     optional MLP head, one hidden layer over the same normed state).
  *
  * Also here: the attention-based key token selection of Sec. 3.2.1 (the
  * last layer's head-averaged attention weights from oracle_forward, the
@@ -332,6 +333,40 @@ double oracle_score_head(const oracle_model *M, const double *h)
     for (int i = 0; i < H; ++i) no += hn[i] * oracle_bf16_to_f64(M->score_head[(size_t)H + i]);
     free(g); free(hn);
     return yes - no;
+}
+
+/*
+ * The lightweight MLP scoring head of Sec. 3.2.3, s = MLP(h_score), whose
+ * shape the paper does not give: here one hidden layer of width d,
+ *   s = sum_j w2[j] * act(sum_i W1[j][i] * hn[i] + b1[j]) + b2,
+ * hn = RMSNorm(h) * g_final (the score token's final state), W1 [d][H],
+ * b1 [d] and w2 [d] bf16, b2 fp64; act: 0 ReLU, 1 GELU (erf form), 2 SiLU,
+ * 3 tanh.
+ */
+double oracle_mlp_head(const oracle_model *M, const double *h, int d, const uint16_t *W1, const uint16_t *b1,
+                       const uint16_t *w2, double b2, int act)
+{
+    const int H = M->hidden;
+    double *g = (double *)malloc(sizeof(double) * (size_t)H);
+    double *xs = (double *)malloc(sizeof(double) * (size_t)H);
+    if (!g || !xs || d < 1 || act < 0 || act > 3) { free(g); free(xs); return NAN; }
+    widen(M->final_norm, H, g);
+    oracle_rmsnorm(h, g, H, M->rms_eps, xs);
+    double s = b2;
+    for (int j = 0; j < d; ++j) {
+        double z = oracle_bf16_to_f64(b1[j]);
+        for (int i = 0; i < H; ++i) z += oracle_bf16_to_f64(W1[(size_t)j * H + i]) * xs[i];
+        double a;
+        switch (act) {
+            case 0: a = z > 0.0 ? z : 0.0; break;
+            case 1: a = 0.5 * z * (1.0 + erf(z / sqrt(2.0))); break;
+            case 2: a = oracle_silu(z); break;
+            default: a = tanh(z); break;
+        }
+        s += oracle_bf16_to_f64(w2[j]) * a;
+    }
+    free(g); free(xs);
+    return s;
 }
 
 /* Embedding lookup of n token ids into x[n][H]. */

@@ -45,6 +45,8 @@ MUTANTS = [
     ("topk_ties_to_higher", "return (x->idx > y->idx) - (x->idx < y->idx);", "return (x->idx < y->idx) - (x->idx > y->idx);"),
     ("probs_average_over_kv_heads", "row[i] += pw[i] / (double)Hq;", "row[i] += pw[i] / (double)Hkv;"),
     ("probs_key_count", "Kall + (size_t)kvh * S * D, m + t + 1, D,", "Kall + (size_t)kvh * S * D, m + t, D,"),
+    ("mlp_bias_dropped", "double z = oracle_bf16_to_f64(b1[j]);", "double z = 0.0;"),
+    ("mlp_gelu_tanh_form", "a = 0.5 * z * (1.0 + erf(z / sqrt(2.0)));", "a = 0.5 * z * (1.0 + tanh(z / sqrt(2.0)));"),
 ]
 
 

@@ -377,3 +377,37 @@ def test_attention_weights_rows_causal_and_consistent_with_outputs():
     V = np.concatenate([pv[L, :, 0], out["v"][L, :, 0]], 0)  # [m + T, D]
     head_mean = out["attn"][L].reshape(T, shape.n_q_heads, D).mean(1)
     np.testing.assert_allclose(P @ V, head_mean, rtol=1e-11, atol=1e-13)
+
+
+# ------------------------------------------------------- MLP scoring head (Sec. 3.2.3)
+
+def _mlp_head(d, H, seed, act, std=0.05):
+    rng = np.random.default_rng(seed)
+    bf = lambda a: torch.tensor(a, dtype=torch.float32).to(torch.bfloat16)
+    return {"w1": bf(rng.normal(0, std, size=(d, H))), "b1": bf(rng.normal(0, 0.1, size=d)),
+            "w2": bf(rng.normal(0, 0.1, size=d)), "b2": 0.25, "act": act}
+
+
+@pytest.mark.parametrize("act", [0, 1, 2, 3])
+def test_mlp_head_matches_torch_composition(act):
+    om, w = tiny_model(seed=12)
+    head = _mlp_head(24, TINY.hidden, 12, act)
+    h = np.random.default_rng(12).normal(size=TINY.hidden)
+    hn = F.rms_norm(torch.tensor(h), (TINY.hidden,), torch.tensor(f64(w["final_norm"])), eps=TINY.rms_eps)
+    z = torch.tensor(f64(head["w1"])) @ hn + torch.tensor(f64(head["b1"]))
+    a = [torch.relu, lambda x: F.gelu(x, approximate="none"), F.silu, torch.tanh][act](z)
+    want = float(torch.tensor(f64(head["w2"])) @ a + head["b2"])
+    assert abs(om.mlp_head(h, head) - want) <= 1e-12 * max(1.0, abs(want))
+
+
+def test_mlp_head_identity_closed_form():
+    # W1 = I, b1 = 0, ReLU, w2 = 1, b2 = 0: the sum of the positive normed components
+    om, w = tiny_model(seed=13)
+    H = TINY.hidden
+    eye = torch.eye(H, dtype=torch.bfloat16)
+    head = {"w1": eye, "b1": torch.zeros(H, dtype=torch.bfloat16), "w2": torch.ones(H, dtype=torch.bfloat16),
+            "b2": 0.0, "act": 0}
+    h = np.random.default_rng(13).normal(size=H)
+    g = f64(w["final_norm"])
+    hn = h / math.sqrt(np.mean(h * h) + TINY.rms_eps) * g
+    assert abs(om.mlp_head(h, head) - np.sum(np.maximum(hn, 0.0))) <= 1e-12
