@@ -107,6 +107,19 @@ DOPR_API dopr_status dopr_model_create(const dopr_model_config *cfg, dopr_model 
 DOPR_API dopr_status dopr_model_put_weight(dopr_model *model, int32_t kind, int32_t layer, const void *src,
                                   int64_t n_elems, int32_t src_on_device);
 
+/*
+ * Replace the yes/no score rows by the paper's lightweight MLP head on the
+ * score token's state (Sec. 3.2.3, s = MLP(h_score); its shape is not given):
+ * one hidden layer of `width` units over hn = RMSNorm(h) * final_norm,
+ *   s = sum_j w2[j] * act(W1[j] . hn + b1[j]) + b2,
+ * W1 bf16 [width][hidden], b1 and w2 bf16 [width]; activation 0 ReLU,
+ * 1 GELU (erf form), 2 SiLU, 3 tanh.  src_on_device != 0: device pointers.
+ * width == 0 restores the yes/no rows.  Synchronous.
+ * Errors: INVALID_ARG, OUT_OF_MEMORY, CUDA.
+ */
+DOPR_API dopr_status dopr_model_set_mlp_head(dopr_model *model, int32_t width, int32_t activation, const void *w1,
+                                            const void *b1, const void *w2, float b2, int32_t src_on_device);
+
 /* Release a model and its device memory.  NULL is accepted. */
 DOPR_API dopr_status dopr_model_destroy(dopr_model *model);
 

@@ -141,6 +141,7 @@ void free_model(Model* m) {
   dev_free(m->embed); dev_free(m->attn_norm); dev_free(m->w_qkv); dev_free(m->q_norm); dev_free(m->k_norm);
   dev_free(m->w_o); dev_free(m->mlp_norm); dev_free(m->w_gu); dev_free(m->w_down); dev_free(m->final_norm);
   dev_free(m->score_head); dev_free(m->rope);
+  dev_free(m->mlp_w1); dev_free(m->mlp_b1); dev_free(m->mlp_w2);
   free_workspace(m->ws);
   for (cudaEvent_t e : m->prof.events) cudaEventDestroy(e);
   m->prof.events.clear();
@@ -754,10 +755,20 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
                            [&] { return launch_gemm(EPI_RESID_ADD, w.tm_act, m->tm_down[l], pd, sms, st); }));
     }
     if (scoring) {
-      CUDA_TRY(prof_launch(m, K_SCORE, 1, 4.0 * H * (s1 - s0), (s1 - s0) * (H * 4.0 + 4.0), st, [&] {
-        return launch_score(w.r_s, H, w.tok_off, t0, s0, s1, 1, w.perm, m->final_norm, m->score_head, c.rms_eps,
-                            d_scores, st);
-      }));
+      if (m->mlp_width > 0) {
+        const double wd = m->mlp_width;
+        CUDA_TRY(prof_launch(m, K_SCORE, 1, 2.0 * H * wd * (s1 - s0), (s1 - s0) * (H * 4.0 + 4.0) + wd * H * 2.0, st,
+                             [&] {
+                               return launch_score_mlp(w.r_s, H, w.tok_off, t0, s0, s1, 1, w.perm, m->final_norm,
+                                                       c.rms_eps, m->mlp_width, m->mlp_act, m->mlp_w1, m->mlp_b1,
+                                                       m->mlp_w2, m->mlp_b2, d_scores, st);
+                             }));
+      } else {
+        CUDA_TRY(prof_launch(m, K_SCORE, 1, 4.0 * H * (s1 - s0), (s1 - s0) * (H * 4.0 + 4.0), st, [&] {
+          return launch_score(w.r_s, H, w.tok_off, t0, s0, s1, 1, w.perm, m->final_norm, m->score_head, c.rms_eps,
+                              d_scores, st);
+        }));
+      }
     } else if (sel) {  // final states of the selected rows: the representations C_d
       SelectArgs sa{};
       sa.tok_off = w.tok_off;
@@ -977,6 +988,32 @@ dopr_status dopr_model_put_weight(dopr_model* m, int32_t kind, int32_t layer, co
     if (e != cudaSuccess) return fail(DOPR_ERR_CUDA, "weight upload failed: %s", cudaGetErrorString(e));
   }
   m->have[(size_t)kind * c.n_layers + l] = 1;
+  return DOPR_OK;
+}
+
+dopr_status dopr_model_set_mlp_head(dopr_model* m, int32_t width, int32_t activation, const void* w1, const void* b1,
+                                    const void* w2, float b2, int32_t src_on_device) {
+  g_last_error.clear();
+  if (!m) return fail(DOPR_ERR_INVALID_ARG, "model is NULL");
+  if (width < 0 || width > 16384) return fail(DOPR_ERR_INVALID_ARG, "width %d outside [0, 16384]", width);
+  if (activation < 0 || activation > 3) return fail(DOPR_ERR_INVALID_ARG, "activation %d outside [0, 3]", activation);
+  CUDA_TRY(cudaSetDevice(m->device));
+  dev_free(m->mlp_w1); dev_free(m->mlp_b1); dev_free(m->mlp_w2);
+  m->mlp_w1 = m->mlp_b1 = m->mlp_w2 = nullptr;
+  m->mlp_width = 0;
+  if (width == 0) return DOPR_OK;  // back to the yes/no rows
+  if (!w1 || !b1 || !w2) return fail(DOPR_ERR_INVALID_ARG, "NULL head weight");
+  const int H = m->cfg.hidden;
+  STATUS_TRY(dev_alloc(&m->mlp_w1, (size_t)width * H));
+  STATUS_TRY(dev_alloc(&m->mlp_b1, (size_t)width));
+  STATUS_TRY(dev_alloc(&m->mlp_w2, (size_t)width));
+  const cudaMemcpyKind kind = src_on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+  CUDA_TRY(cudaMemcpy(m->mlp_w1, w1, sizeof(bf16) * (size_t)width * H, kind));
+  CUDA_TRY(cudaMemcpy(m->mlp_b1, b1, sizeof(bf16) * (size_t)width, kind));
+  CUDA_TRY(cudaMemcpy(m->mlp_w2, w2, sizeof(bf16) * (size_t)width, kind));
+  m->mlp_width = width;
+  m->mlp_act = activation;
+  m->mlp_b2 = b2;
   return DOPR_OK;
 }
 

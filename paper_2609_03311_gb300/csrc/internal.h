@@ -146,6 +146,12 @@ struct Model {
   f16* w_down = nullptr;       // [L][H][F]
   bf16* final_norm = nullptr;  // [H]
   bf16* score_head = nullptr;  // [2][H]
+  // optional MLP scoring head (replaces the yes/no rows when mlp_width > 0)
+  int mlp_width = 0, mlp_act = 0;
+  bf16* mlp_w1 = nullptr;  // [width][H]
+  bf16* mlp_b1 = nullptr;  // [width]
+  bf16* mlp_w2 = nullptr;  // [width]
+  float mlp_b2 = 0.f;
   float2* rope = nullptr;      // [max_position][64] (cos, sin)
   std::vector<uint8_t> have;   // [kind * L + layer]
   std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
@@ -209,6 +215,9 @@ cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0
                          cudaStream_t st);
 // Compact the score-token rows of sorted pairs [p_begin, p_end): dst_r[i] = r[row(i)] (H floats) and
 // dst_ss[i] = ss[row(i)] (parts floats), row(i) = tok_off[p_begin+i+1]-1-tok0.
+cudaError_t launch_score_mlp(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end,
+                             int compact, const int32_t* perm, const bf16* gain, float eps, int width, int act,
+                             const bf16* w1, const bf16* b1, const bf16* w2, float b2, float* scores, cudaStream_t st);
 cudaError_t launch_gather_score_rows(const float* r, const float* ss, int H, int parts, const int32_t* tok_off,
                                      int tok0, int p_begin, int p_end, float* dst_r, float* dst_ss, cudaStream_t st);
 // [m][Hkv][128] bf16 -> [Hkv][m][128] fp16 for K and V; *range |= 1 when a value

@@ -95,6 +95,59 @@ __global__ void __launch_bounds__(ROW_WARPS * 32)
   if (lane == 0) scores[perm[s]] = yes - no;
 }
 
+// MLP scoring head (Sec. 3.2.3): one CTA per pair.  hn = RMSNorm(row) * g in
+// shared memory; each warp takes hidden units j = warp, warp + 8, ...: z = W1[j] . hn
+// + b1[j], act(z) * w2[j] summed; the block sum + b2 is the score.
+constexpr int MLP_THREADS = 256;
+__device__ __forceinline__ float head_act(float z, int act) {
+  switch (act) {
+    case 0: return fmaxf(z, 0.f);
+    case 1: return 0.5f * z * (1.f + erff(z * 0.70710678118654752f));
+    case 2: return z / (1.f + expf(-z));
+    default: return tanhf(z);
+  }
+}
+__global__ void __launch_bounds__(MLP_THREADS)
+    k_score_mlp(const float* __restrict__ r, int H, const int32_t* __restrict__ tok_off, int tok0, int p_begin,
+                int compact, const int32_t* __restrict__ perm, const bf16* __restrict__ gain, float eps, int width,
+                int act, const bf16* __restrict__ w1, const bf16* __restrict__ b1, const bf16* __restrict__ w2,
+                float b2, float* __restrict__ scores) {
+  extern __shared__ float hn[];  // [H], then 32 partial sums
+  float* red = hn + H;
+  const int s = p_begin + blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t row = compact ? s - p_begin : tok_off[s + 1] - 1 - tok0;
+  const float* x = r + row * H;
+  float ss = 0.f;
+  for (int c = threadIdx.x; c < H; c += blockDim.x) ss += x[c] * x[c];
+  ss = warp_sum(ss);
+  if (lane == 0) red[warp] = ss;
+  __syncthreads();
+  float tot = 0.f;
+  for (int w = 0; w < MLP_THREADS / 32; ++w) tot += red[w];
+  const float inv = rsqrtf(tot / static_cast<float>(H) + eps);
+  for (int c = threadIdx.x; c < H; c += blockDim.x) hn[c] = x[c] * inv * __bfloat162float(gain[c]);
+  __syncthreads();
+  float part = 0.f;
+  for (int j = warp; j < width; j += MLP_THREADS / 32) {
+    const bf16* wr = w1 + static_cast<int64_t>(j) * H;
+    float z = 0.f;
+    for (int c = lane * 2; c < H; c += 64) {
+      const float2 wv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(wr + c));
+      z += wv.x * hn[c] + wv.y * hn[c + 1];
+    }
+    z = warp_sum(z) + __bfloat162float(b1[j]);
+    part += head_act(z, act) * __bfloat162float(w2[j]);
+  }
+  __syncthreads();
+  if (lane == 0) red[warp] = part;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float sc = b2;
+    for (int w = 0; w < MLP_THREADS / 32; ++w) sc += red[w];
+    scores[perm[s]] = sc;
+  }
+}
+
 // One warp per pair: copy its score-token row of r (and of the partial sums) to row i.
 __global__ void __launch_bounds__(ROW_WARPS * 32)
     k_gather_score_rows(const float* __restrict__ r, const float* __restrict__ ss, int H, int parts,
@@ -198,6 +251,15 @@ cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0
   if (p_end <= p_begin) return cudaSuccess;
   k_score<<<blocks_for(p_end - p_begin), ROW_WARPS * 32, 0, st>>>(r, H, tok_off, tok0, p_begin, p_end, compact, perm,
                                                                   gain, head, eps, scores);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_score_mlp(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end,
+                             int compact, const int32_t* perm, const bf16* gain, float eps, int width, int act,
+                             const bf16* w1, const bf16* b1, const bf16* w2, float b2, float* scores, cudaStream_t st) {
+  if (p_end <= p_begin) return cudaSuccess;
+  k_score_mlp<<<p_end - p_begin, MLP_THREADS, (H + 32) * sizeof(float), st>>>(
+      r, H, tok_off, tok0, p_begin, compact, perm, gain, eps, width, act, w1, b1, w2, b2, scores);
   return cudaGetLastError();
 }
 

@@ -76,6 +76,7 @@ def load():
         "dopr_build_prefixes": ([P, P, i32, P, P, P, i32, P], i32),
         "dopr_debug_store_read": ([P, i64, i32, P, P], i32),
         "dopr_select_prefix_inputs": ([P, i32, P, P, i32, i32, P, P, P, P], i32),
+        "dopr_model_set_mlp_head": ([P, i32, i32, P, P, P, ctypes.c_float, i32], i32),
         "dopr_last_error": ([], ctypes.c_char_p),
         "dopr_version": ([], ctypes.c_char_p),
     }
@@ -204,6 +205,18 @@ class Store:
             self.close()
         except Exception:
             pass
+
+
+def set_mlp_head(model: Model, head: dict | None):
+    """Use the MLP scoring head {w1 bf16 [d, H], b1 bf16 [d], w2 bf16 [d], b2 float,
+    act 0..3} instead of the yes/no rows; None restores the rows."""
+    if head is None:
+        _check(load().dopr_model_set_mlp_head(model._h, 0, 0, None, None, None, 0.0, 0))
+        return
+    w1, b1, w2 = (head[k].contiguous() for k in ("w1", "b1", "w2"))
+    assert w1.dtype == b1.dtype == w2.dtype == torch.bfloat16
+    _check(load().dopr_model_set_mlp_head(model._h, int(w1.shape[0]), int(head["act"]), _ptr(w1), _ptr(b1), _ptr(w2),
+                                          float(head["b2"]), int(w1.is_cuda)))
 
 
 def build_prefixes(model: Model, store: Store, doc_ids, x_offsets, x: torch.Tensor, stream=None):
