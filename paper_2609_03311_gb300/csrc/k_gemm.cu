@@ -112,6 +112,11 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
       const int hc = nb * BN + hh * 128;  // first output column of this head
       const bool rope = (EPI == EPI_QKV) && hc < p.q_cols + p.k_cols;
       if (rope) {
+        // positions of the 8 rows this lane rotates (transposed layout below), loaded
+        // before the sum-of-squares pass so their latency overlaps it
+        int pos_i[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) pos_i[i] = p.tok_pos[min(row0 + i * 4 + (lane >> 3), p.M - 1)];
         // per-head RMSNorm of the row-scaled values: sum of squares in the row layout
         float ss = 0.f;
 #pragma unroll 1
@@ -129,15 +134,26 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
         // stores are contiguous 8-lane row segments
         const int w4 = (lane & 7) * 4;
         float inv_i[8];
-        int pos_i[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int r = i * 4 + (lane >> 3);
-          inv_i[i] = __shfl_sync(0xffffffffu, inv_row, r);
-          pos_i[i] = row0 + r < p.M ? p.tok_pos[row0 + r] : 0;
-        }
+        for (int i = 0; i < 8; ++i) inv_i[i] = __shfl_sync(0xffffffffu, inv_row, i * 4 + (lane >> 3));
 #pragma unroll 1
         for (int c = 0; c < 64; c += 32) {
+          // the rows' (cos, sin) for frequencies c+w4 .. +3, loaded first (rows past M
+          // read position 0's entries and are not stored) so the loads overlap the
+          // accumulator reads below
+          float4 c01[8], c23[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float4* cs = reinterpret_cast<const float4*>(p.rope + static_cast<int64_t>(pos_i[i]) * 64 + c + w4);
+            c01[i] = cs[0];
+            c23[i] = cs[1];
+          }
+          float g1[4], g2[4];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            g1[k] = __bfloat162float(wgt[c + w4 + k]);
+            g2[k] = __bfloat162float(wgt[64 + c + w4 + k]);
+          }
           float4 x1[8], x2[8];
 #pragma unroll
           for (int half = 0; half < 2; ++half) {
@@ -159,19 +175,12 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
             }
             __syncwarp();
           }
-          float g1[4], g2[4];
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            g1[k] = __bfloat162float(wgt[c + w4 + k]);
-            g2[k] = __bfloat162float(wgt[64 + c + w4 + k]);
-          }
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             const int r = i * 4 + (lane >> 3);
             if (row0 + r < p.M) {
-              const float4* cs = reinterpret_cast<const float4*>(p.rope + static_cast<int64_t>(pos_i[i]) * 64 + c + w4);
-              const float4 c01 = cs[0], c23 = cs[1];  // (cos, sin) for frequencies c+w4 .. +3
-              const float cosv[4] = {c01.x, c01.z, c23.x, c23.z}, sinv[4] = {c01.y, c01.w, c23.y, c23.w};
+              const float cosv[4] = {c01[i].x, c01[i].z, c23[i].x, c23[i].z};
+              const float sinv[4] = {c01[i].y, c01[i].w, c23[i].y, c23[i].w};
               const float a[4] = {x1[i].x, x1[i].y, x1[i].z, x1[i].w}, b[4] = {x2[i].x, x2[i].y, x2[i].z, x2[i].w};
               float y1[4], y2[4];
 #pragma unroll
