@@ -64,12 +64,31 @@ __device__ __forceinline__ void tile_coords(int t, int m_tiles, int n_tiles, int
 
 __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + __expf(-x)); }
 
-// RMSNorm factor of a row from its partial sums of squares (fixed summation order).
+// RMSNorm factor of a row from its partial sums of squares, added in index
+// order.  When the count allows, the partials arrive as independent 16-byte
+// loads (up to 32 in flight) instead of one dependent load per partial.
 __device__ __forceinline__ float norm_factor(const float* ss, int parts, const GemmParams& p, int row) {
   if (!ss) return 1.f;
   const float* s = ss + static_cast<int64_t>(min(row, p.M - 1)) * parts;
   float t = 0.f;
-  for (int i = 0; i < parts; ++i) t += s[i];
+  if ((parts & 3) == 0) {
+    for (int i = 0; i < parts; i += 32) {
+      float4 v[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        v[q] = i + 4 * q < parts ? __ldg(reinterpret_cast<const float4*>(s + i) + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        if (i + 4 * q < parts) {
+          t += v[q].x;
+          t += v[q].y;
+          t += v[q].z;
+          t += v[q].w;
+        }
+    }
+  } else {
+    for (int i = 0; i < parts; ++i) t += s[i];
+  }
   return rsqrtf(t / static_cast<float>(p.norm_dim) + p.eps);
 }
 // Consumer-side row scale: the operand was written as r * g * rs(ss_pre).
@@ -222,10 +241,12 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
     float* res = reinterpret_cast<float*>(p.out);
     const int w4 = (lane & 7) * 4;
     float ss[8], pre[8];
+    // each lane fetches its own row's previous norm factor; the row layout below takes them by shuffle
+    const float pre_mine = p.xn_out ? norm_factor(p.ss_pre, p.ss_pre_parts, p, row) : 1.f;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       ss[i] = 0.f;
-      pre[i] = p.xn_out ? norm_factor(p.ss_pre, p.ss_pre_parts, p, row0 + i * 4 + (lane >> 3)) : 1.f;
+      pre[i] = __shfl_sync(0xffffffffu, pre_mine, i * 4 + (lane >> 3));
     }
     auto rrow = [&](int i, int c) {
       return reinterpret_cast<float4*>(res + static_cast<int64_t>(row0 + i * 4 + (lane >> 3)) * p.ld_out + nb * BN +
