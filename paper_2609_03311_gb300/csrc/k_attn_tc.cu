@@ -16,20 +16,21 @@
 //
 // Persistent CTAs, one per SM, warp-specialised:
 //   warp 0    TMA producer: the Q tile (two stages), the tile's key blocks of
-//             64 columns into a K ring and a V ring (three stages each) --
+//             64 columns into a K ring (five stages) and a V ring (three) --
 //             prefix blocks from the store pool in 64-row boxes, own-key
 //             segments from the packed QKV buffer in 16-row boxes;
 //   warp 1    MMA issuer: S = Q K^T for every key block into the unit's TMEM
-//             region (fp32, up to 256 columns), then O = P V block by block, V
-//             read as an MN-major operand, over the region's first 128 columns
-//             once the softmax has read them; S of the next unit goes in
-//             before P V of this one;
+//             region (fp32, up to 256 columns), then O = P V block by block
+//             with P read from TMEM and V from shared memory as an MN-major
+//             operand, into the region's upper 128 columns (over S blocks 2
+//             and 3, when the unit has them, once the softmax has read them);
+//             S of the next unit goes in before P V of this one;
 //   warps 2-9 two softmax/epilogue warpgroups taking alternate units, one
 //             thread per tile row (its TMEM lane): an exact two-pass softmax
 //             over the row's S (the maximum over the visible keys, then exp2
 //             and fixed-shape 16-key sums added in key order), P written as
-//             fp16 into the warpgroup's two-stage ring in the UMMA K-major
-//             layout, and after the last P V step O / sum as fp16.
+//             fp16 into TMEM over S columns already read, and after the last
+//             P V step O / sum as fp16, staged per warp for whole-line stores.
 // The exact maximum, the in-order sum and the aligned own segments make every
 // row's result independent of how the batch was cut into tiles.
 // Every wait is bounded; a CTA that gives up lets its copies and MMAs land and
@@ -47,35 +48,37 @@ constexpr int TILE_M = 128;
 constexpr int KBLK = 64;  // key columns per block
 constexpr int GROUP_ROWS = 16;
 constexpr int NSLOT = 2;  // tiles in flight: one softmax warpgroup and one TMEM region each
-constexpr int Q_STAGES = 2, KV_STAGES = 3, P_STAGES = 2;  // P stages per slot
+constexpr int Q_STAGES = 2, K_STAGES = 5, V_STAGES = 3;
 constexpr int Q_HALF = TILE_M * 128;    // 128 rows x 64 16-bit elements
 constexpr int Q_BYTES = 2 * Q_HALF;     // 32 KB
 constexpr int KV_HALF = KBLK * 128;     // 64 rows x 64 elements
 constexpr int KV_BYTES = 2 * KV_HALF;   // 16 KB
 constexpr int P_BYTES = TILE_M * 128;   // 128 rows x 64 keys
 constexpr int GROUP_BYTES = 2 * GROUP_ROWS * 128;
+constexpr int EP_WARP_BYTES = 32 * 128;  // one warp's 32 rows x 64 fp16 columns of O on the way out
 constexpr int THREADS = 64 + NSLOT * 128;
-// TMEM: slot s owns columns [256 s, 256 s + 256) -- S, and once the softmax has read
-// S's first 128 columns, O over them
-constexpr uint32_t TMEM_COLS = 512, SLOT_COLS = 256;
+constexpr int MAX_BLOCKS = ATTN_TC_MAX_KEYS / KBLK;  // 4
+// TMEM region of a slot (256 columns): S at [0, 64 nb); P of block j, fp16, at
+// [32 j, 32 j + 32) over S columns the softmax has read; O at [128, 256), over
+// S blocks 2 and 3 when the unit has them.
+constexpr uint32_t TMEM_COLS = 512, SLOT_COLS = 256, O_COL = 128;
 
 constexpr int OFF_Q = 0;
 constexpr int OFF_K = OFF_Q + Q_STAGES * Q_BYTES;
-constexpr int OFF_V = OFF_K + KV_STAGES * KV_BYTES;
-constexpr int OFF_P = OFF_V + KV_STAGES * KV_BYTES;
-constexpr int OFF_BAR = OFF_P + NSLOT * P_STAGES * P_BYTES;
+constexpr int OFF_V = OFF_K + K_STAGES * KV_BYTES;
+constexpr int OFF_EP = OFF_V + V_STAGES * KV_BYTES;
+constexpr int OFF_BAR = OFF_EP + NSLOT * 4 * EP_WARP_BYTES;
 constexpr int BAR_Q_FULL = 0, BAR_Q_EMPTY = BAR_Q_FULL + Q_STAGES;
-constexpr int BAR_K_FULL = BAR_Q_EMPTY + Q_STAGES, BAR_K_EMPTY = BAR_K_FULL + KV_STAGES;
-constexpr int BAR_V_FULL = BAR_K_EMPTY + KV_STAGES, BAR_V_EMPTY = BAR_V_FULL + KV_STAGES;
-constexpr int BAR_P_FULL = BAR_V_EMPTY + KV_STAGES;           // [slot][stage]
-constexpr int BAR_P_EMPTY = BAR_P_FULL + NSLOT * P_STAGES;    // [slot][stage]
-constexpr int BAR_S_FULL = BAR_P_EMPTY + NSLOT * P_STAGES;    // [slot]: S complete
-constexpr int BAR_R_FREE = BAR_S_FULL + NSLOT;                // [slot]: the region's O read out
-constexpr int BAR_O_FULL = BAR_R_FREE + NSLOT;                // [slot]: O complete
+constexpr int BAR_K_FULL = BAR_Q_EMPTY + Q_STAGES, BAR_K_EMPTY = BAR_K_FULL + K_STAGES;
+constexpr int BAR_V_FULL = BAR_K_EMPTY + K_STAGES, BAR_V_EMPTY = BAR_V_FULL + V_STAGES;
+constexpr int BAR_P_FULL = BAR_V_EMPTY + V_STAGES;             // [slot][block]: P of the block is in TMEM
+constexpr int BAR_S_FULL = BAR_P_FULL + NSLOT * MAX_BLOCKS;    // [slot]: S complete
+constexpr int BAR_R_FREE = BAR_S_FULL + NSLOT;                 // [slot]: the region's O read out
+constexpr int BAR_O_FULL = BAR_R_FREE + NSLOT;                 // [slot]: O complete
 constexpr int BAR_DRAIN = BAR_O_FULL + NSLOT, N_BARS = BAR_DRAIN + 1;
+static_assert(BAR_V_FULL + V_STAGES <= 32, "the producer tracks the barriers it arms in one 32-bit mask");
 constexpr int SMEM_BYTES = 1024 + OFF_BAR + N_BARS * 8 + 16;
 static_assert(SMEM_BYTES <= 227 * 1024, "shared memory budget");
-static_assert(BAR_V_FULL + KV_STAGES <= 32, "producer arm mask");
 
 constexpr uint32_t IDESC_S = umma_idesc_f16(TILE_M, KBLK);
 constexpr uint32_t IDESC_O = umma_idesc_f16_bmn(TILE_M, HEAD_DIM);
@@ -169,6 +172,31 @@ __device__ __forceinline__ float exp_chunk(uint32_t (&v)[32], uint32_t mask, flo
   return sum;
 }
 
+// The same P values, packed as fp16 pairs (key 2i in the low half of pk[i]) for a
+// TMEM store; returns sum + the two 16-column partial sums in column order.
+__device__ __forceinline__ float exp_pack(uint32_t (&v)[32], uint32_t mask, float scale_log2, float mxs, float sum,
+                                          uint32_t (&pk)[16]) {
+#pragma unroll
+  for (int e = 0; e < 32; ++e) {
+    const float x = ex2_approx(fmaf(__uint_as_float(v[e]), scale_log2, -mxs));
+    v[e] = __float_as_uint((mask >> e) & 1u ? x : 0.f);
+  }
+#pragma unroll
+  for (int i = 0; i < 16; ++i) pk[i] = pack_f16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+#pragma unroll
+  for (int gidx = 0; gidx < 2; ++gidx) {
+    float t[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) t[i] = __uint_as_float(v[16 * gidx + 2 * i]) + __uint_as_float(v[16 * gidx + 2 * i + 1]);
+#pragma unroll
+    for (int w2 = 4; w2 >= 1; w2 >>= 1)
+#pragma unroll
+      for (int i = 0; i < w2; ++i) t[i] = t[2 * i] + t[2 * i + 1];
+    sum += t[0];
+  }
+  return sum;
+}
+
 __device__ __forceinline__ void zero_chunk(uint8_t* prow, int half, int r) {
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
@@ -183,7 +211,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t s0 = smem_u32(smem);
-  const uint32_t sQ = s0 + OFF_Q, sK = s0 + OFF_K, sV = s0 + OFF_V, sP = s0 + OFF_P;
+  const uint32_t sQ = s0 + OFF_Q, sK = s0 + OFF_K, sV = s0 + OFF_V;
   auto bar = [&](int i) { return s0 + OFF_BAR + 8u * static_cast<uint32_t>(i); };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + OFF_BAR + N_BARS * 8);
 
@@ -199,16 +227,15 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_init(bar(BAR_Q_FULL + i), 1);
       mbar_init(bar(BAR_Q_EMPTY + i), 1);
     }
-    for (int i = 0; i < KV_STAGES; ++i) {
+    for (int i = 0; i < K_STAGES; ++i) {
       mbar_init(bar(BAR_K_FULL + i), 1);
       mbar_init(bar(BAR_K_EMPTY + i), 1);
+    }
+    for (int i = 0; i < V_STAGES; ++i) {
       mbar_init(bar(BAR_V_FULL + i), 1);
       mbar_init(bar(BAR_V_EMPTY + i), 1);
     }
-    for (int i = 0; i < NSLOT * P_STAGES; ++i) {
-      mbar_init(bar(BAR_P_FULL + i), 4);
-      mbar_init(bar(BAR_P_EMPTY + i), 1);
-    }
+    for (int i = 0; i < NSLOT * MAX_BLOCKS; ++i) mbar_init(bar(BAR_P_FULL + i), 4);
     for (int i = 0; i < NSLOT; ++i) {
       mbar_init(bar(BAR_S_FULL + i), 1);
       mbar_init(bar(BAR_R_FREE + i), 4);
@@ -285,7 +312,7 @@ __global__ void __launch_bounds__(THREADS, 1)
               }
             }
           }
-          r.next(KV_STAGES);
+          r.next(kv ? V_STAGES : K_STAGES);
         }
         return true;
       };
@@ -312,7 +339,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       // ======================= MMA issuer: an event loop over non-blocking barrier tests.
       // P V blocks of unit ip go in as soon as their P and V are there; S blocks of
       // unit is (at most one unit ahead) as soon as Q, the slot's region and K are.
-      Ring rq, rk, rv, rp[NSLOT];
+      Ring rq, rk, rv;
+      uint32_t ppar = 0;            // bit slot * MAX_BLOCKS + j: parity of the next P_FULL completion
       int is = 0, js = 0, nbs = 0;  // S: unit, next block, blocks
       bool s_open = false;          // unit is's Q and region are in hand
       int ip = 0, jp = 0;           // P V: unit, next block
@@ -320,36 +348,35 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = true;
       while (ip < n_local) {
         bool prog = false;
-        // ---- O = P V of unit ip, whose S is complete
+        // ---- O = P V of unit ip, whose S is complete; P is read from TMEM
         if (ip < is) {
           const int slot = ip & 1;
           const int n_keys = a.tiles[unit_of(ip) / a.Hkv].n_keys;
           const int nbp = (n_keys + KBLK - 1) / KBLK;
-          Ring& r = rp[slot];
+          auto p_ready = [&](int j) {
+            return mbar_test(bar(BAR_P_FULL + slot * MAX_BLOCKS + j), (ppar >> (slot * MAX_BLOCKS + j)) & 1u);
+          };
           while (jp < nbp) {
-            bool ready = mbar_test(bar(BAR_P_FULL + slot * P_STAGES + r.stage), r.phase);
-            if (ready && jp == 0 && nbp > 1) {  // O overwrites S columns 0..127: the softmax must be past block 1
-              Ring r1 = r;
-              r1.next(P_STAGES);
-              ready = mbar_test(bar(BAR_P_FULL + slot * P_STAGES + r1.stage), r1.phase);
-            }
+            bool ready = p_ready(jp);
+            // O (columns 128..255) covers S blocks 2 and 3: with more than two blocks the
+            // softmax must be past its last S read, i.e. the last block's P is in
+            if (ready && jp == 0 && nbp > 2) ready = p_ready(nbp - 1);
             if (!ready || !mbar_test(bar(BAR_V_FULL + rv.stage), rv.phase)) break;
             tc_fence_after();
             const int steps = min(KBLK, n_keys - jp * KBLK) / 16;  // only rows the producer loaded
-            const uint64_t pd = umma_desc_sw128(sP + (slot * P_STAGES + r.stage) * P_BYTES);
+            const uint32_t pcol = tmem + slot * SLOT_COLS + 32 * jp;  // 16 keys = 8 columns per step
             for (int kk = 0; kk < steps; ++kk)
-              umma_f16(tmem + slot * SLOT_COLS, pd + (kk * 32) / 16,
-                       umma_desc_sw128_mn(sV + rv.stage * KV_BYTES + kk * 2048, KV_HALF, 1024), IDESC_O,
-                       (jp | kk) != 0);
-            umma_commit(bar(BAR_P_EMPTY + slot * P_STAGES + r.stage));
+              umma_f16_ts(tmem + slot * SLOT_COLS + O_COL, pcol + 8 * kk,
+                          umma_desc_sw128_mn(sV + rv.stage * KV_BYTES + kk * 2048, KV_HALF, 1024), IDESC_O,
+                          (jp | kk) != 0);
             umma_commit(bar(BAR_V_EMPTY + rv.stage));
-            r.next(P_STAGES);
-            rv.next(KV_STAGES);
+            rv.next(V_STAGES);
             ++jp;
             prog = true;
           }
           if (jp == nbp) {
             umma_commit(bar(BAR_O_FULL + slot));
+            for (int j = 0; j < nbp; ++j) ppar ^= 1u << (slot * MAX_BLOCKS + j);  // each block's barrier completed once
             ++ip;
             jp = 0;
             prog = true;
@@ -376,7 +403,7 @@ __global__ void __launch_bounds__(THREADS, 1)
               umma_f16(tmem + slot * SLOT_COLS + js * KBLK, qd + ((ks >> 2) * Q_HALF + (ks & 3) * 32) / 16,
                        kd + ((ks >> 2) * KV_HALF + (ks & 3) * 32) / 16, IDESC_S, ks > 0);
             umma_commit(bar(BAR_K_EMPTY + rk.stage));
-            rk.next(KV_STAGES);
+            rk.next(K_STAGES);
             ++js;
             prog = true;
           }
@@ -409,8 +436,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int jj = r % TT;  // this row's token within the tile (its q head is r / TT)
     const uint32_t trow = tmem + slot * SLOT_COLS + (static_cast<uint32_t>(quarter * 32) << 16);
     const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(HEAD_DIM));
-    uint8_t* prow0 = smem + OFF_P + slot * P_STAGES * P_BYTES + r * 128;
-    Ring rp;
+    uint8_t* stg = smem + OFF_EP + (slot * 4 + quarter) * EP_WARP_BYTES;  // this warp's staging lines
     for (int i = slot, k = 0; i < n_local; i += NSLOT, ++k) {
       const uint32_t par = static_cast<uint32_t>(k & 1);
       const int u = unit_of(i);
@@ -454,80 +480,75 @@ __global__ void __launch_bounds__(THREADS, 1)
         mx = fmaxf(mx, masked_max32(v, vis_mask(c0)));
       }
       const float mxs = (mx == -INFINITY) ? 0.f : mx * scale_log2;
-      // ---- pass 2: P = 2^((s - max) * scale) per 64-key block; the sum adds
+      // ---- pass 2: P = 2^((s - max) * scale) per 64-key block, as fp16 into TMEM
+      // columns [32 j, 32 j + 32) (S columns this pass has read); the sum adds
       // fixed-shape 16-key partial sums in key order
       float sum = 0.f;
-      bool ok = true;
-      for (int c0 = 0; c0 < ncol; c0 += KBLK) {
-        if (!mbar_wait(bar(BAR_P_EMPTY + slot * P_STAGES + rp.stage), rp.phase ^ 1u, a.err, WAIT_TIMEOUT_NS)) {
-          ok = false;
-          break;
-        }
-        uint8_t* prow = prow0 + rp.stage * P_BYTES;
+      for (int c0 = 0, j = 0; c0 < ncol; c0 += KBLK, ++j) {
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
           const int cb = c0 + 32 * half;
+          uint32_t pk[16];
           if (chunk_live(cb)) {
             uint32_t v[32];
             tmem_ld32(trow + cb, v);
             tmem_ld_wait();
-            sum = exp_chunk(v, vis_mask(cb), scale_log2, mxs, sum, prow, half, r);
+            sum = exp_pack(v, vis_mask(cb), scale_log2, mxs, sum, pk);
           } else {
-            zero_chunk(prow, half, r);
+#pragma unroll
+            for (int q = 0; q < 16; ++q) pk[q] = 0u;
           }
+          tmem_st16(trow + 32 * j + 16 * half, pk);
         }
-        fence_proxy_async_smem();  // generic-proxy P writes -> visible to the tensor core
-        tc_fence_before();         // this block's S reads precede the O writes that may follow
+        tmem_st_wait();
+        tc_fence_before();  // this block's S reads and P writes precede the MMAs that follow
         __syncwarp();
-        if (lane == 0) mbar_arrive(bar(BAR_P_FULL + slot * P_STAGES + rp.stage));
-        rp.next(P_STAGES);
+        if (lane == 0) mbar_arrive(bar(BAR_P_FULL + slot * MAX_BLOCKS + j));
       }
-      if (!ok) break;
-      // ---- epilogue: O / sum -> fp16 at (token, q head g * G + hh).  The rows go
-      // through this warp's own lines of the slot's two P stages (idle once P V is
-      // done): row rr of the warp at stage rr / 16, 256 bytes per row, 16-byte
-      // chunks swizzled by the row; then each store instruction writes two whole
-      // 256-byte rows.
+      // ---- epilogue: O / sum -> fp16 at (token, q head g * G + hh), 64 columns at a
+      // time through this warp's staging lines (128 bytes per row, 16-byte chunks
+      // swizzled by the row), each store instruction writing four 128-byte row pieces
       if (!mbar_wait(bar(BAR_O_FULL + slot), par, a.err, WAIT_TIMEOUT_NS)) break;
       tc_fence_after();
       const float inv = sum > 0.f ? 1.f / sum : 0.f;
-      uint8_t* stg = smem + OFF_P + slot * P_STAGES * P_BYTES + quarter * 32 * 128;
-      auto stg_row = [&](int rr) { return stg + (rr >> 4) * P_BYTES + (rr & 15) * 256; };
 #pragma unroll 1
-      for (int c0 = 0; c0 < HEAD_DIM; c0 += 32) {
-        uint32_t v[32];
-        tmem_ld32(trow + c0, v);
-        tmem_ld_wait();
+      for (int h = 0; h < 2; ++h) {
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const uint32_t* x = v + 8 * q;
-          uint4 o;
-          o.x = pack_f16x2(__uint_as_float(x[0]) * inv, __uint_as_float(x[1]) * inv);
-          o.y = pack_f16x2(__uint_as_float(x[2]) * inv, __uint_as_float(x[3]) * inv);
-          o.z = pack_f16x2(__uint_as_float(x[4]) * inv, __uint_as_float(x[5]) * inv);
-          o.w = pack_f16x2(__uint_as_float(x[6]) * inv, __uint_as_float(x[7]) * inv);
-          const int chunk = c0 / 8 + q;
-          *reinterpret_cast<uint4*>(stg_row(lane) + ((chunk ^ (lane & 7)) << 4)) = o;
+        for (int c2 = 0; c2 < 2; ++c2) {
+          uint32_t v[32];
+          tmem_ld32(trow + O_COL + 64 * h + 32 * c2, v);
+          tmem_ld_wait();
+          if (h == 1 && c2 == 1) {  // O is out of TMEM: the region is free
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(BAR_R_FREE + slot));
+          }
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const uint32_t* x = v + 8 * q;
+            uint4 o;
+            o.x = pack_f16x2(__uint_as_float(x[0]) * inv, __uint_as_float(x[1]) * inv);
+            o.y = pack_f16x2(__uint_as_float(x[2]) * inv, __uint_as_float(x[3]) * inv);
+            o.z = pack_f16x2(__uint_as_float(x[4]) * inv, __uint_as_float(x[5]) * inv);
+            o.w = pack_f16x2(__uint_as_float(x[6]) * inv, __uint_as_float(x[7]) * inv);
+            const int chunk = c2 * 4 + q;
+            *reinterpret_cast<uint4*>(stg + lane * 128 + ((chunk ^ (lane & 7)) << 4)) = o;
+          }
         }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(bar(BAR_R_FREE + slot));  // O is out of TMEM: the region is free
-      {
-        const int half = lane >> 4, ch = lane & 15;
-#pragma unroll 4
-        for (int it = 0; it < 16; ++it) {
-          const int rr = 2 * it + half;
+        __syncwarp();
+#pragma unroll
+        for (int it = 0; it < 8; ++it) {
+          const int rr = it * 4 + (lane >> 3), ch = lane & 7;
           const int row = quarter * 32 + rr;  // tile row
           const int j2 = row % TT;
           if (j2 < n_tok) {
-            const uint4 x = *reinterpret_cast<const uint4*>(stg_row(rr) + ((ch ^ (rr & 7)) << 4));
+            const uint4 x = *reinterpret_cast<const uint4*>(stg + rr * 128 + ((ch ^ (rr & 7)) << 4));
             *reinterpret_cast<uint4*>(a.out + static_cast<int64_t>(tp->tok_begin + j2) * a.ld_out +
-                                      (g * G + row / TT) * HEAD_DIM + ch * 8) = x;
+                                      (g * G + row / TT) * HEAD_DIM + 64 * h + ch * 8) = x;
           }
         }
+        __syncwarp();  // staging reads finish before the next half's writes
       }
-      __syncwarp();  // staging reads finish before this warp writes P rows of the next unit
     }
   }
 
