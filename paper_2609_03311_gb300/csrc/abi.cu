@@ -368,36 +368,39 @@ struct Plan {
 };
 
 // Attention plan of a call: tensor-core tiles of at most TT tokens -- short ones
-// within ATTN_TC_MAX_KEYS key columns, long ones (pairs whose own keys alone can
-// exceed that) without a key limit -- and, when G gives no tile shape, runs of
-// pairs for the mma.sync kernel.  Tiles keep at most ATTN_TC_MAX_SEGS pairs.
+// within ATTN_TC_MAX_KEYS key columns, long ones (whose first token alone needs
+// more) without a key limit -- and, when G gives no tile shape, runs of pairs for
+// the mma.sync kernel.  Tiles keep at most ATTN_TC_MAX_SEGS pairs.
 struct AttnPlanner {
   int TT = 0;
   std::vector<AttnTile> tiles, ltiles;
   std::vector<AttnItem> litems;
 
   // The sorted pairs [pb, pe) of one document (token offsets `to`, t0 the chunk's first token).
+  // Each tile takes up to TT consecutive tokens (at most ATTN_TC_MAX_SEGS pairs).  It is a
+  // tensor-core tile when its key columns fit ATTN_TC_MAX_KEYS -- the tile is cut where the
+  // next token would overflow -- and a long tile, with no key limit, when not even its first
+  // token fits.  Both kernels compute a row identically, so which one a row lands in does not
+  // change its result.
   void add(const int32_t* to, int32_t t0, int32_t pb, int32_t pe, int32_t slot, int32_t m, int64_t pool_base) {
     auto c16 = [](int x) { return (x + 15) & ~15; };
-    auto fits = [&](int32_t p) { return attn_tc_pair_fits(m, to[p + 1] - to[p]); };
     const int pre64 = ((m + 63) / 64) * 64;
-    int32_t p = pb;
-    while (p < pe) {
-      int32_t q = p + 1;
-      if (TT == 0) {
-        while (q < pe && q - p < ATTN_MAX_PAIRS) ++q;
+    if (TT == 0) {
+      for (int32_t p = pb; p < pe;) {
+        const int32_t q = std::min(pe, p + ATTN_MAX_PAIRS);
         litems.push_back(AttnItem{p, q, slot, m});
         p = q;
-        continue;
       }
-      const bool is_long = !fits(p);
-      while (q < pe && fits(q) != is_long) ++q;  // a run of pairs of one kind
-      std::vector<AttnTile>& out = is_long ? ltiles : tiles;
-      const int32_t end = to[q] - t0;
-      int32_t tok = to[p] - t0, pf = p;
-      while (tok < end) {
-        while (to[pf + 1] - t0 <= tok) ++pf;
-        int32_t n = 0, closed = 0, keys = 0, pp = pf;
+      return;
+    }
+    const int32_t end = to[pe] - t0;
+    int32_t tok = to[pb] - t0, pf = pb;
+    while (tok < end) {
+      while (to[pf + 1] - t0 <= tok) ++pf;
+      // the tokens [tok, tok + n) a tile takes, and its key columns
+      auto grow = [&](bool limit_keys, int32_t& keys) {
+        int32_t n = 0, closed = 0, pp = pf;
+        keys = 0;
         while (n < TT && tok + n < end) {
           const int32_t t = tok + n;
           while (to[pp + 1] - t0 <= t) {  // pair pp lies wholly in the tile: its full segment
@@ -405,24 +408,28 @@ struct AttnPlanner {
             ++pp;
           }
           const int32_t k = pre64 + closed + c16(t - (to[pp] - t0) + 1);
-          if ((!is_long && k > ATTN_TC_MAX_KEYS) || pp - pf >= ATTN_TC_MAX_SEGS) break;
+          if ((limit_keys && k > ATTN_TC_MAX_KEYS) || pp - pf >= ATTN_TC_MAX_SEGS) break;
           keys = k;
           ++n;
         }
-        AttnTile tl{};
-        tl.pool_base = pool_base;
-        tl.tok_begin = tok;
-        tl.n_tok = n;
-        tl.m = m;
-        tl.n_keys = keys;
-        for (int32_t sp = pf; to[sp] - t0 < tok + n; ++sp) {
-          const int32_t ps = to[sp] - t0, nvis = std::min(to[sp + 1] - t0, tok + n) - ps;
-          tl.seg[tl.n_seg++] = (int32_t)(((uint32_t)nvis << 16) | (uint16_t)(int16_t)(ps - tok));
-        }
-        out.push_back(tl);
-        tok += n;
+        return n;
+      };
+      int32_t keys = 0;
+      int32_t n = grow(true, keys);
+      const bool is_long = n == 0;
+      if (is_long) n = grow(false, keys);
+      AttnTile tl{};
+      tl.pool_base = pool_base;
+      tl.tok_begin = tok;
+      tl.n_tok = n;
+      tl.m = m;
+      tl.n_keys = keys;
+      for (int32_t sp = pf; to[sp] - t0 < tok + n; ++sp) {
+        const int32_t ps = to[sp] - t0, nvis = std::min(to[sp + 1] - t0, tok + n) - ps;
+        tl.seg[tl.n_seg++] = (int32_t)(((uint32_t)nvis << 16) | (uint16_t)(int16_t)(ps - tok));
       }
-      p = q;
+      (is_long ? ltiles : tiles).push_back(tl);
+      tok += n;
     }
   }
   void close_chunk(Plan& plan) const {

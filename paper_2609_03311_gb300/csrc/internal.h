@@ -256,10 +256,6 @@ struct AttnTcArgs {
 };
 // Q rows per head in a 128-row tile; 0 when the group size does not divide 128 into boxes of >= 8 rows.
 inline int attn_tc_rows_per_head(int G) { return (G >= 1 && G <= 16 && 128 % G == 0) ? 128 / G : 0; }
-// Whether a pair of T tokens (query + score token) on a prefix of m keys fits one tile's key budget.
-inline bool attn_tc_pair_fits(int m, int T) {
-  return ((m + 63) / 64) * 64 + ((T + 15) / 16) * 16 <= ATTN_TC_MAX_KEYS;
-}
 cudaError_t attn_tc_setup();
 // tm_q: the chunk's packed QKV buffer, box 64 columns x (128 / G) rows; tm_kv: the same
 // buffer, box 64 x 16; tm_pool: the store pool, box 64 x 64 (all fp16, 128-byte swizzle).

@@ -53,7 +53,6 @@ constexpr int Q_HALF = TILE_M * 128;    // 128 rows x 64 16-bit elements
 constexpr int Q_BYTES = 2 * Q_HALF;     // 32 KB
 constexpr int KV_HALF = KBLK * 128;     // 64 rows x 64 elements
 constexpr int KV_BYTES = 2 * KV_HALF;   // 16 KB
-constexpr int P_BYTES = TILE_M * 128;   // 128 rows x 64 keys
 constexpr int GROUP_BYTES = 2 * GROUP_ROWS * 128;
 constexpr int EP_WARP_BYTES = 32 * 128;  // one warp's 32 rows x 64 fp16 columns of O on the way out
 constexpr int THREADS = 64 + NSLOT * 128;
@@ -139,41 +138,10 @@ __device__ __forceinline__ float masked_max32(const uint32_t (&v)[32], uint32_t 
   return t[0];
 }
 
-// P for 32 columns: 2^(s * scale - mxs) where the mask bit is set, else 0, stored
-// as fp16 into 16-byte chunks 4*half .. 4*half+3 of the row's 128-byte P line
-// (128-byte swizzle).  Returns sum + the two 16-column partial sums, each a
-// fixed pairwise tree, added in column order.
-__device__ __forceinline__ float exp_chunk(uint32_t (&v)[32], uint32_t mask, float scale_log2, float mxs, float sum,
-                                           uint8_t* prow, int half, int r) {
-#pragma unroll
-  for (int e = 0; e < 32; ++e) {  // in place: v now holds the 32 P values
-    const float x = ex2_approx(fmaf(__uint_as_float(v[e]), scale_log2, -mxs));
-    v[e] = __float_as_uint((mask >> e) & 1u ? x : 0.f);
-  }
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int chunk = half * 4 + q;
-    const uint32_t* x = v + 8 * q;
-    *reinterpret_cast<uint4*>(prow + ((chunk ^ (r & 7)) << 4)) = make_uint4(
-        pack_f16x2(__uint_as_float(x[0]), __uint_as_float(x[1])), pack_f16x2(__uint_as_float(x[2]), __uint_as_float(x[3])),
-        pack_f16x2(__uint_as_float(x[4]), __uint_as_float(x[5])), pack_f16x2(__uint_as_float(x[6]), __uint_as_float(x[7])));
-  }
-#pragma unroll
-  for (int gidx = 0; gidx < 2; ++gidx) {
-    float t[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) t[i] = __uint_as_float(v[16 * gidx + 2 * i]) + __uint_as_float(v[16 * gidx + 2 * i + 1]);
-#pragma unroll
-    for (int w2 = 4; w2 >= 1; w2 >>= 1)
-#pragma unroll
-      for (int i = 0; i < w2; ++i) t[i] = t[2 * i] + t[2 * i + 1];
-    sum += t[0];
-  }
-  return sum;
-}
-
-// The same P values, packed as fp16 pairs (key 2i in the low half of pk[i]) for a
-// TMEM store; returns sum + the two 16-column partial sums in column order.
+// P for 32 columns: 2^(s * scale - mxs) where the mask bit is set, else 0, packed
+// as fp16 pairs (key 2i in the low half of pk[i]) for a TMEM store.  Returns
+// sum + the two 16-column partial sums, each a fixed pairwise tree, added in
+// column order.
 __device__ __forceinline__ float exp_pack(uint32_t (&v)[32], uint32_t mask, float scale_log2, float mxs, float sum,
                                           uint32_t (&pk)[16]) {
 #pragma unroll
@@ -195,14 +163,6 @@ __device__ __forceinline__ float exp_pack(uint32_t (&v)[32], uint32_t mask, floa
     sum += t[0];
   }
   return sum;
-}
-
-__device__ __forceinline__ void zero_chunk(uint8_t* prow, int half, int r) {
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int chunk = half * 4 + q;
-    *reinterpret_cast<uint4*>(prow + ((chunk ^ (r & 7)) << 4)) = make_uint4(0, 0, 0, 0);
-  }
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
@@ -566,19 +526,21 @@ __global__ void __launch_bounds__(THREADS, 1)
 // longest prefixes with long queries, uncompressed documents).  One unit at a
 // time per CTA, one softmax warpgroup, the keys in 128-column chunks through
 // two S buffers: pass A computes S chunk by chunk for the exact row maximum,
-// pass B computes each chunk again, writes P and accumulates O = P V in its own
+// pass B computes each chunk again, writes P as fp16 into a four-stage TMEM
+// ring and accumulates O = P V (P from TMEM, as in the short kernel) in its own
 // 128 TMEM columns.  The row results are the short kernel's: the same maximum,
 // the same 16-key sums in key order, the same MMA steps.
 namespace lt {
-constexpr int Q_STAGES = 2, K_STAGES = 3, V_STAGES = 3, P_STAGES = 2;
+constexpr int Q_STAGES = 2, K_STAGES = 5, V_STAGES = 3, P_STAGES = 4;
 constexpr int CH = 128;  // key columns per S chunk
 constexpr int THREADS = 64 + 128;
-constexpr uint32_t O_COL = 0, S_COL = 128;  // S buffer b at S_COL + CH * b
+// TMEM: O at [0, 128), S buffer b at S_COL + CH b, P stage s (64 keys as fp16) at P_COL + 32 s
+constexpr uint32_t O_COL = 0, S_COL = 128, P_COL = 384;
 constexpr int OFF_Q = 0;
 constexpr int OFF_K = OFF_Q + Q_STAGES * Q_BYTES;
 constexpr int OFF_V = OFF_K + K_STAGES * KV_BYTES;
-constexpr int OFF_P = OFF_V + V_STAGES * KV_BYTES;
-constexpr int OFF_BAR = OFF_P + P_STAGES * P_BYTES;
+constexpr int OFF_EP = OFF_V + V_STAGES * KV_BYTES;
+constexpr int OFF_BAR = OFF_EP + 4 * EP_WARP_BYTES;
 constexpr int B_Q_FULL = 0, B_Q_EMPTY = B_Q_FULL + Q_STAGES;
 constexpr int B_K_FULL = B_Q_EMPTY + Q_STAGES, B_K_EMPTY = B_K_FULL + K_STAGES;
 constexpr int B_V_FULL = B_K_EMPTY + K_STAGES, B_V_EMPTY = B_V_FULL + V_STAGES;
@@ -588,6 +550,7 @@ constexpr int B_O_FULL = B_S_FREE + 2, B_O_FREE = B_O_FULL + 1, B_DRAIN = B_O_FR
 constexpr int SMEM_BYTES = 1024 + OFF_BAR + N_BARS * 8 + 16;
 static_assert(SMEM_BYTES <= 227 * 1024, "shared memory budget");
 static_assert(B_V_FULL + V_STAGES <= 32, "producer arm mask");
+static_assert(P_COL + 32 * P_STAGES <= TMEM_COLS, "P ring inside the allocation");
 }  // namespace lt
 
 __global__ void __launch_bounds__(lt::THREADS, 1)
@@ -596,7 +559,7 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t s0 = smem_u32(smem);
-  const uint32_t sQ = s0 + lt::OFF_Q, sK = s0 + lt::OFF_K, sV = s0 + lt::OFF_V, sP = s0 + lt::OFF_P;
+  const uint32_t sQ = s0 + lt::OFF_Q, sK = s0 + lt::OFF_K, sV = s0 + lt::OFF_V;
   auto bar = [&](int i) { return s0 + lt::OFF_BAR + 8u * static_cast<uint32_t>(i); };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + lt::OFF_BAR + lt::N_BARS * 8);
 
@@ -768,10 +731,10 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
             if (!wait(lt::B_P_FULL + rp.stage, rp.phase) || !wait(lt::B_V_FULL + rv.stage, rv.phase)) break;
             tc_fence_after();
             const int steps = min(KBLK, n_keys - j * KBLK) / 16;
-            const uint64_t pd = umma_desc_sw128(sP + rp.stage * P_BYTES);
+            const uint32_t pcol = tmem + lt::P_COL + 32 * rp.stage;  // 16 keys = 8 columns per step
             const uint64_t vd = umma_desc_sw128_mn(sV + rv.stage * KV_BYTES, KV_HALF, 1024);
             for (int kk = 0; kk < steps; ++kk)
-              umma_f16(tmem + lt::O_COL, pd + (kk * 32) / 16, vd + (kk * 2048) / 16, IDESC_O, (j | kk) != 0);
+              umma_f16_ts(tmem + lt::O_COL, pcol + 8 * kk, vd + (kk * 2048) / 16, IDESC_O, (j | kk) != 0);
             umma_commit(bar(lt::B_P_EMPTY + rp.stage));
             umma_commit(bar(lt::B_V_EMPTY + rv.stage));
             rp.next(lt::P_STAGES);
@@ -792,8 +755,8 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
     const int r = quarter * 32 + lane;
     const int jj = r % TT;  // this row's token within the tile (its q head is r / TT)
     const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(HEAD_DIM));
-    uint8_t* prow0 = smem + lt::OFF_P + r * 128;
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    uint8_t* stg = smem + lt::OFF_EP + quarter * EP_WARP_BYTES;  // this warp's staging lines
     Ring rp;
     uint32_t cc = 0;
     bool ok = true;
@@ -861,20 +824,23 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
             ok = false;
             break;
           }
-          uint8_t* prow = prow0 + rp.stage * P_BYTES;
 #pragma unroll
           for (int hf = 0; hf < 2; ++hf) {
             const int cb = j * KBLK + 32 * hf;
+            uint32_t pk[16];
             if (chunk_live(cb)) {
               uint32_t v[32];
               tmem_ld32(lane_base + lt::S_COL + lt::CH * buf + (cb - c * lt::CH), v);
               tmem_ld_wait();
-              sum = exp_chunk(v, vis_mask(cb), scale_log2, mxs, sum, prow, hf, r);
+              sum = exp_pack(v, vis_mask(cb), scale_log2, mxs, sum, pk);
             } else {
-              zero_chunk(prow, hf, r);
+#pragma unroll
+              for (int q = 0; q < 16; ++q) pk[q] = 0u;
             }
+            tmem_st16(lane_base + lt::P_COL + 32 * rp.stage + 16 * hf, pk);
           }
-          fence_proxy_async_smem();
+          tmem_st_wait();
+          tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(bar(lt::B_P_FULL + rp.stage));
           rp.next(lt::P_STAGES);
@@ -886,46 +852,48 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
         ++cc;
       }
       if (!ok) break;
-      // ---- epilogue: O / sum -> fp16, staged through this warp's own P lines
+      // ---- epilogue: O / sum -> fp16, 64 columns at a time through this warp's staging lines
       if (!mbar_wait(bar(lt::B_O_FULL), static_cast<uint32_t>(i) & 1u, a.err, WAIT_TIMEOUT_NS)) break;
       tc_fence_after();
       const float inv = sum > 0.f ? 1.f / sum : 0.f;
-      uint8_t* stg = smem + lt::OFF_P + quarter * 32 * 128;
-      auto stg_row = [&](int rr) { return stg + (rr >> 4) * P_BYTES + (rr & 15) * 256; };
 #pragma unroll 1
-      for (int c0 = 0; c0 < HEAD_DIM; c0 += 32) {
-        uint32_t v[32];
-        tmem_ld32(lane_base + lt::O_COL + c0, v);
-        tmem_ld_wait();
+      for (int h = 0; h < 2; ++h) {
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const uint32_t* x = v + 8 * q;
-          uint4 o;
-          o.x = pack_f16x2(__uint_as_float(x[0]) * inv, __uint_as_float(x[1]) * inv);
-          o.y = pack_f16x2(__uint_as_float(x[2]) * inv, __uint_as_float(x[3]) * inv);
-          o.z = pack_f16x2(__uint_as_float(x[4]) * inv, __uint_as_float(x[5]) * inv);
-          o.w = pack_f16x2(__uint_as_float(x[6]) * inv, __uint_as_float(x[7]) * inv);
-          *reinterpret_cast<uint4*>(stg_row(lane) + (((c0 / 8 + q) ^ (lane & 7)) << 4)) = o;
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(bar(lt::B_O_FREE));
-      {
-        const int half = lane >> 4, ch = lane & 15;
-#pragma unroll 4
-        for (int it = 0; it < 16; ++it) {
-          const int rr = 2 * it + half;
-          const int row = quarter * 32 + rr;
-          const int j2 = row % TT;
-          if (j2 < n_tok) {
-            const uint4 x = *reinterpret_cast<const uint4*>(stg_row(rr) + ((ch ^ (rr & 7)) << 4));
-            *reinterpret_cast<uint4*>(a.out + static_cast<int64_t>(tp->tok_begin + j2) * a.ld_out +
-                                      (g * G + row / TT) * HEAD_DIM + ch * 8) = x;
+        for (int c2 = 0; c2 < 2; ++c2) {
+          uint32_t v[32];
+          tmem_ld32(lane_base + lt::O_COL + 64 * h + 32 * c2, v);
+          tmem_ld_wait();
+          if (h == 1 && c2 == 1) {  // O is out of TMEM
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(lt::B_O_FREE));
+          }
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const uint32_t* x = v + 8 * q;
+            uint4 o;
+            o.x = pack_f16x2(__uint_as_float(x[0]) * inv, __uint_as_float(x[1]) * inv);
+            o.y = pack_f16x2(__uint_as_float(x[2]) * inv, __uint_as_float(x[3]) * inv);
+            o.z = pack_f16x2(__uint_as_float(x[4]) * inv, __uint_as_float(x[5]) * inv);
+            o.w = pack_f16x2(__uint_as_float(x[6]) * inv, __uint_as_float(x[7]) * inv);
+            const int chunk = c2 * 4 + q;
+            *reinterpret_cast<uint4*>(stg + lane * 128 + ((chunk ^ (lane & 7)) << 4)) = o;
           }
         }
+        __syncwarp();
+#pragma unroll
+        for (int it = 0; it < 8; ++it) {
+          const int rr = it * 4 + (lane >> 3), ch = lane & 7;
+          const int row = quarter * 32 + rr;  // tile row
+          const int j2 = row % TT;
+          if (j2 < n_tok) {
+            const uint4 x = *reinterpret_cast<const uint4*>(stg + rr * 128 + ((ch ^ (rr & 7)) << 4));
+            *reinterpret_cast<uint4*>(a.out + static_cast<int64_t>(tp->tok_begin + j2) * a.ld_out +
+                                      (g * G + row / TT) * HEAD_DIM + 64 * h + ch * 8) = x;
+          }
+        }
+        __syncwarp();  // staging reads finish before the next half's writes
       }
-      __syncwarp();
     }
   }
 

@@ -198,6 +198,34 @@ def test_batch_order_and_chunking_do_not_change_scores():
     np.testing.assert_array_equal(singles, base[:8])
 
 
+def test_rows_split_between_short_and_long_tiles_are_batch_invariant():
+    # Prefixes of 100-200 keys with queries of 20-250 tokens: a long pair's early tiles fit
+    # the tensor-core kernel's 256 key columns and its later ones take the long-tile kernel,
+    # and which tile (so which kernel) a row lands in depends on the other pairs of its
+    # document in the batch.  The rows' results must not.
+    rig = Rig(SMALL_G4, {0: 128, 1: 100, 2: 200}, seed=12)
+    pairs = synth.random_pairs(24, 3, 20, 250, SMALL_G4.vocab, seed=12)
+    qo, qt, di = pairs["q_offsets"], pairs["q_tokens"], pairs["doc_ids"]
+    lens = np.diff(qo)
+    assert lens.max() + 128 > 256 and lens.min() + 100 < 256
+    base = rig.score(pairs)
+    idx = sorted({int(np.argmax(lens)), int(np.argmin(lens)), 3})
+    ref = rig.oracle(pairs, idx)
+    assert np.max(np.abs(base[idx] - ref)) <= TOL, np.max(np.abs(base[idx] - ref))
+
+    def sub(sel):
+        return {"q_offsets": np.concatenate([[0], np.cumsum(lens[sel])]).astype(np.int32),
+                "q_tokens": np.concatenate([qt[qo[p]:qo[p + 1]] for p in sel]).astype(np.int32),
+                "doc_ids": di[sel]}
+
+    perm = np.random.default_rng(12).permutation(24)
+    np.testing.assert_array_equal(rig.score(sub(perm)), base[perm])
+    odd = np.arange(1, 24, 2)
+    np.testing.assert_array_equal(rig.score(sub(odd)), base[odd])
+    for p in (int(np.argmax(lens)), 0, 7):
+        np.testing.assert_array_equal(rig.score(sub(np.array([p]))), base[p:p + 1])
+
+
 def test_device_io_matches_host_io():
     rig = Rig(SMALL_G2, {0: 64, 1: 100}, seed=8)
     pairs = synth.random_pairs(30, 2, 0, 40, SMALL_G2.vocab, seed=8)
