@@ -265,6 +265,27 @@ DOPR_API dopr_status dopr_debug_pack_plan(dopr_model *model, dopr_store *store, 
                                  int32_t *tok_pos, int32_t *tok_id, int32_t *tok_pair);
 
 /*
+ * The attention tile plan of one document's run of pairs, computed on the
+ * host exactly as dopr_score plans it (no device work: usable without a GPU),
+ * for testing the tiling rule of the prefix-plus-causal attention (Sec. 3.4).
+ *   m              the document's prefix length (keys), >= 0;
+ *   rows_per_tile  tokens per tile (128 / G for G q heads per kv head), 1..128;
+ *   n_pairs        pairs of the run, >= 1; tok_len [n_pairs] int32 >= 1: the
+ *                  packed tokens (query + score token) of each pair, laid out
+ *                  consecutively in this order;
+ *   out            [max_tiles][24] int32, caller-owned; tile t, in token order:
+ *                  {kind (0 = tensor-core tile of at most 256 key columns, 1 =
+ *                  long tile), tok_begin, n_tok, n_keys, n_seg, 0, 0, 0,
+ *                  seg[0..15]}, seg[s] = (visible tokens << 16) | (uint16_t)
+ *                  (first token of the pair - tok_begin), one per pair the tile
+ *                  touches, in pair order.
+ * Returns the number of tiles (>= 1), or -DOPR_ERR_INVALID_ARG for bad
+ * arguments or when max_tiles is too small (nothing is written then).
+ */
+DOPR_API int32_t dopr_debug_attention_plan(int32_t m, int32_t rows_per_tile, int32_t n_pairs, const int32_t *tok_len,
+                                           int32_t max_tiles, int32_t *out);
+
+/*
  * The dense projection kernel alone, for testing: C = A * B^T with A fp16
  * [M][K], B fp16 [N][K] (IEEE half, device pointers), fp32 accumulation.
  *   epilogue 0: out fp16 [M][N] = C

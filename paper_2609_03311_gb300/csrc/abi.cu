@@ -1439,6 +1439,46 @@ dopr_status dopr_debug_pack_plan(dopr_model* m, dopr_store* s, int32_t n, const 
   return map_device_error(*w.h_err);
 }
 
+int32_t dopr_debug_attention_plan(int32_t m, int32_t rows_per_tile, int32_t n_pairs, const int32_t* tok_len,
+                                  int32_t max_tiles, int32_t* out) {
+  g_last_error.clear();
+  if (m < 0 || rows_per_tile < 1 || rows_per_tile > 128 || n_pairs < 1 || !tok_len || max_tiles < 0 || !out) {
+    fail(DOPR_ERR_INVALID_ARG, "bad attention-plan arguments");
+    return -DOPR_ERR_INVALID_ARG;
+  }
+  std::vector<int32_t> to(n_pairs + 1, 0);
+  for (int32_t p = 0; p < n_pairs; ++p) {
+    if (tok_len[p] < 1 || to[p] > INT32_MAX - tok_len[p]) {
+      fail(DOPR_ERR_INVALID_ARG, "tok_len[%d] must be >= 1", p);
+      return -DOPR_ERR_INVALID_ARG;
+    }
+    to[p + 1] = to[p] + tok_len[p];
+  }
+  AttnPlanner pl;
+  pl.TT = rows_per_tile;
+  pl.add(to.data(), 0, 0, n_pairs, 0, m, 0);
+  std::vector<std::pair<int32_t, const AttnTile*>> all;  // (kind, tile) in token order
+  for (const AttnTile& t : pl.tiles) all.push_back({0, &t});
+  for (const AttnTile& t : pl.ltiles) all.push_back({1, &t});
+  std::sort(all.begin(), all.end(), [](const auto& a, const auto& b) { return a.second->tok_begin < b.second->tok_begin; });
+  if ((int64_t)all.size() > max_tiles) {
+    fail(DOPR_ERR_INVALID_ARG, "the plan has %zu tiles, max_tiles is %d", all.size(), max_tiles);
+    return -DOPR_ERR_INVALID_ARG;
+  }
+  for (size_t i = 0; i < all.size(); ++i) {
+    const AttnTile& t = *all[i].second;
+    int32_t* o = out + 24 * i;
+    o[0] = all[i].first;
+    o[1] = t.tok_begin;
+    o[2] = t.n_tok;
+    o[3] = t.n_keys;
+    o[4] = t.n_seg;
+    o[5] = o[6] = o[7] = 0;
+    for (int j = 0; j < ATTN_TC_MAX_SEGS; ++j) o[8 + j] = j < t.n_seg ? t.seg[j] : 0;
+  }
+  return (int32_t)all.size();
+}
+
 dopr_status dopr_debug_gemm(int32_t M, int32_t N, int32_t K, const void* A, const void* B, void* out,
                             int32_t epilogue, void* cuda_stream) {
   g_last_error.clear();

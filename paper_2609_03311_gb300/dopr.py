@@ -75,6 +75,7 @@ def load():
         "dopr_profile_read": ([P, P, i32], i32),
         "dopr_build_prefixes": ([P, P, i32, P, P, P, i32, P], i32),
         "dopr_debug_store_read": ([P, i64, i32, P, P], i32),
+        "dopr_debug_attention_plan": ([i32, i32, i32, P, i32, P], i32),
         "dopr_select_prefix_inputs": ([P, i32, P, P, i32, i32, P, P, P, P], i32),
         "dopr_model_set_mlp_head": ([P, i32, i32, P, P, P, ctypes.c_float, i32], i32),
         "dopr_last_error": ([], ctypes.c_char_p),
@@ -282,6 +283,18 @@ def pack_plan(model: Model, store: Store, q_offsets, q_tokens, doc_ids) -> dict:
                                        _ptr(perm), _ptr(tok_off), _ptr(tok_pos), _ptr(tok_id), _ptr(tok_pair)))
     return {"perm": perm[:n], "tok_off": tok_off, "tok_pos": tok_pos[:T], "tok_id": tok_id[:T],
             "tok_pair": tok_pair[:T]}
+
+
+def attention_plan(m: int, rows_per_tile: int, tok_len) -> np.ndarray:
+    """The attention tiles of one document's run of pairs (host-only, no GPU):
+    int32 [n_tiles, 24] rows {kind, tok_begin, n_tok, n_keys, n_seg, 0, 0, 0, seg[16]}."""
+    tl = _host(tok_len, np.int32)
+    cap = int(tl.sum()) + 1
+    out = np.zeros((cap, 24), np.int32)
+    n = load().dopr_debug_attention_plan(int(m), int(rows_per_tile), len(tl), _ptr(tl), cap, _ptr(out))
+    if n < 0:
+        _check(-n)
+    return out[:n]
 
 
 def gemm(A: torch.Tensor, B: torch.Tensor, epilogue: int = EPI_STORE, out: torch.Tensor | None = None):
