@@ -118,24 +118,43 @@ __device__ __forceinline__ void store_words_transposed(const uint32_t* xs, int l
   }
 }
 
+// What an epilogue reads that does not depend on the accumulator: fetched while
+// the tile's main loop still runs, so its load latency is off the epilogue's path.
+struct EpiPre {
+  float scale;  // this thread's row: the consumer row scale (QKV, SwiGLU) or the previous norm factor
+  int pos[8];   // QKV: positions of the 8 rows a lane rotates in the transposed layout
+};
+
+template <int EPI>
+__device__ __forceinline__ void epilogue_prefetch(const GemmParams& p, int mb, int nb, int quarter, int part,
+                                                  int lane, EpiPre& pre) {
+  const int row0 = mb * BM + quarter * 32;
+  if constexpr (EPI == EPI_RESID_ADD) {
+    pre.scale = p.xn_out ? norm_factor(p.ss_pre, p.ss_pre_parts, p, row0 + lane) : 1.f;
+  } else if constexpr (EPI == EPI_STORE) {
+    pre.scale = 1.f;
+  } else {
+    pre.scale = row_scale(p, row0 + lane);
+  }
+  if constexpr (EPI == EPI_QKV) {
+    if (nb * BN + part * 128 < p.q_cols + p.k_cols)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) pre.pos[i] = p.tok_pos[min(row0 + i * 4 + (lane >> 3), p.M - 1)];
+  }
+}
+
 template <int EPI>
 __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t taddr, int mb, int nb, int quarter,
-                                              int part, int lane, uint32_t* xs) {
-  const int row0 = mb * BM + quarter * 32;  // first row of this warp
-  const int row = row0 + lane;              // this thread's row (TMEM lane)
+                                              int part, int lane, uint32_t* xs, const EpiPre& pre) {
+  const int row0 = mb * BM + quarter * 32;  // first row of this warp; lane = row - row0 = TMEM lane
   if constexpr (EPI == EPI_STORE || EPI == EPI_QKV) {
     f16* out = reinterpret_cast<f16*>(p.out);
-    const float rs = row_scale(p, row);
+    const float rs = pre.scale;
     {
       const int hh = part;                 // this warp's 128-column head of the tile
       const int hc = nb * BN + hh * 128;  // first output column of this head
       const bool rope = (EPI == EPI_QKV) && hc < p.q_cols + p.k_cols;
       if (rope) {
-        // positions of the 8 rows this lane rotates (transposed layout below), loaded
-        // before the sum-of-squares pass so their latency overlaps it
-        int pos_i[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) pos_i[i] = p.tok_pos[min(row0 + i * 4 + (lane >> 3), p.M - 1)];
         // per-head RMSNorm of the row-scaled values: sum of squares in the row layout
         float ss = 0.f;
 #pragma unroll 1
@@ -157,13 +176,12 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
         for (int i = 0; i < 8; ++i) inv_i[i] = __shfl_sync(0xffffffffu, inv_row, i * 4 + (lane >> 3));
 #pragma unroll 1
         for (int c = 0; c < 64; c += 32) {
-          // the rows' (cos, sin) for frequencies c+w4 .. +3, loaded first (rows past M
-          // read position 0's entries and are not stored) so the loads overlap the
-          // accumulator reads below
+          // the rows' (cos, sin) for frequencies c+w4 .. +3 (rows past M read position
+          // 0's entries and are not stored), ahead of the accumulator reads below
           float4 c01[8], c23[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
-            const float4* cs = reinterpret_cast<const float4*>(p.rope + static_cast<int64_t>(pos_i[i]) * 64 + c + w4);
+            const float4* cs = reinterpret_cast<const float4*>(p.rope + static_cast<int64_t>(pre.pos[i]) * 64 + c + w4);
             c01[i] = cs[0];
             c23[i] = cs[1];
           }
@@ -240,13 +258,12 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
     // residual values of chunk c+1 are loaded while chunk c is processed.
     float* res = reinterpret_cast<float*>(p.out);
     const int w4 = (lane & 7) * 4;
-    float ss[8], pre[8];
-    // each lane fetches its own row's previous norm factor; the row layout below takes them by shuffle
-    const float pre_mine = p.xn_out ? norm_factor(p.ss_pre, p.ss_pre_parts, p, row) : 1.f;
+    float ss[8], prev[8];
+    // each lane fetched its own row's previous norm factor; the row layout below takes them by shuffle
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       ss[i] = 0.f;
-      pre[i] = __shfl_sync(0xffffffffu, pre_mine, i * 4 + (lane >> 3));
+      prev[i] = __shfl_sync(0xffffffffu, pre.scale, i * 4 + (lane >> 3));
     }
     auto rrow = [&](int i, int c) {
       return reinterpret_cast<float4*>(res + static_cast<int64_t>(row0 + i * 4 + (lane >> 3)) * p.ld_out + nb * BN +
@@ -290,7 +307,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
           *rrow(i, c) = x;
           if (p.xn_out) {
             ss[i] += x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w;
-            const float sc = pre[i];
+            const float sc = prev[i];
             uint2 o;
             o.x = pack_f16x2(x.x * g4.x * sc, x.y * g4.y * sc);
             o.y = pack_f16x2(x.z * g4.z * sc, x.w * g4.w * sc);
@@ -315,7 +332,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
     }
   } else {  // EPI_SWIGLU: columns 0..127 gate, 128..255 up of the same 128 outputs
     f16* out = reinterpret_cast<f16*>(p.out);
-    const float rs = row_scale(p, row);
+    const float rs = pre.scale;
     {
       const int c = part * 64;  // this warp's 64 of the tile's 128 outputs
 #pragma unroll
@@ -466,10 +483,12 @@ __global__ void __launch_bounds__(THREADS, 1)
       tile_coords(t, m_tiles, n_tiles, mb, nb);
       const int acc = local & 1;
       const uint32_t acc_phase = (local >> 1) & 1;
+      EpiPre pre;
+      epilogue_prefetch<EPI>(p, mb, nb, quarter, part, lane, pre);
       if (!mbar_wait(tfull_bar(acc), acc_phase, p.err, p.timeout_ns)) break;
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
-      epilogue_tile<EPI>(p, taddr, mb, nb, quarter, part, lane, xs);
+      epilogue_tile<EPI>(p, taddr, mb, nb, quarter, part, lane, xs, pre);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty_bar(acc));
