@@ -78,6 +78,30 @@ def test_salience_positions_and_states_match_oracle(shape, top_p):
     model.close()
 
 
+def test_selection_at_the_document_length_limit():
+    # a 2,048-token document (the longest the selection accepts) next to a short one
+    shape = SHAPE_G2
+    w = synth.make_weights(shape, seed=44, norms="random")
+    model = dopr.Model(dopr.make_config(shape, max_position=4096), w)
+    om = oracle.OracleModel(oshape(shape), w)
+    lens = [2048, 3]
+    K = 64
+    off, tok, docs = _docs(shape, lens, seed=44)
+    pos, x, u = dopr.select_prefix_inputs(model, off, tok, K, 10 ** 6)
+    for d, ids in enumerate(docs):
+        out = om.forward(om.embed(ids), 0, want_probs=True)
+        ref_u = oracle.salience(out["probs"], 10 ** 6)
+        got_u = u[off[d]:off[d + 1]].astype(np.float64)
+        assert np.all(np.abs(got_u - ref_u) <= _u_tol(ref_u)), (d, float(np.max(np.abs(got_u - ref_u))))
+        k = min(K, len(ids))
+        sel = pos[d, :k]
+        assert np.all(np.diff(sel) > 0) and np.all(pos[d, k:] == -1)
+        rest = np.setdiff1d(np.arange(len(ids)), sel)
+        if len(rest):
+            assert ref_u[rest].max() <= ref_u[sel].min() + 2 * _u_tol(ref_u).max()
+    model.close()
+
+
 def test_select_build_score_pipeline_matches_oracle():
     # offline selection -> prefix build -> online scoring, on both sides from the same positions
     shape = SHAPE
