@@ -531,7 +531,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 // 128 TMEM columns.  The row results are the short kernel's: the same maximum,
 // the same 16-key sums in key order, the same MMA steps.
 namespace lt {
-constexpr int Q_STAGES = 2, K_STAGES = 5, V_STAGES = 3, P_STAGES = 4;
+constexpr int Q_STAGES = 2, K_STAGES = 5, V_STAGES = 4, P_STAGES = 4;
 constexpr int CH = 128;  // key columns per S chunk
 constexpr int THREADS = 64 + 128;
 // TMEM: O at [0, 128), S buffer b at S_COL + CH b, P stage s (64 keys as fp16) at P_COL + 32 s
