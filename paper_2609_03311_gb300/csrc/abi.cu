@@ -583,14 +583,15 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     const double attn_bytes_last = np * 2.0 * Hq * HEAD_DIM * 2 + T * 2.0 * Hkv * HEAD_DIM * 2 +
                                    prefix_rows * Hkv * 2 * HEAD_DIM * 2;
     // this chunk's packed QKV buffer as TMA maps for the tensor-core attention:
-    // Q boxes of 128 / G rows per q head, own-key boxes of 16 rows
+    // Q boxes of 128 / G rows per q head, own-key boxes of 16 and of 64 rows
     const int TT = attn_tc_rows_per_head(Hq / Hkv);
-    CUtensorMap tm_q{}, tm_kv{};
+    CUtensorMap tm_q{}, tm_kv{}, tm_kv64{};
     const int n_tiles = plan.chunk_tile[ci + 1] - plan.chunk_tile[ci];
     const int n_ltiles = plan.chunk_ltile[ci + 1] - plan.chunk_ltile[ci];
     if (n_tiles + n_ltiles > 0 &&
         !(make_tmap_16b_2d(&tm_q, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, TT, true, true) &&
-          make_tmap_16b_2d(&tm_kv, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, 16, true, true)))
+          make_tmap_16b_2d(&tm_kv, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, 16, true, true) &&
+          make_tmap_16b_2d(&tm_kv64, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, 64, true, true)))
       return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for the QKV buffer");
     AttnTcArgs ta{};
     ta.tiles = w.tiles + plan.chunk_tile[ci];
@@ -697,11 +698,11 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
                              cudaError_t e = cudaSuccess;
                              if (!last && ta.n_units > 0) {
                                ta.layer = l;
-                               e = launch_attention_tc(tm_q, tm_kv, s->tm_pool, ta, sms, st);
+                               e = launch_attention_tc(tm_q, tm_kv, tm_kv64, s->tm_pool, ta, sms, st);
                              }
                              if (e == cudaSuccess && !last && tl.n_units > 0) {
                                tl.layer = l;
-                               e = launch_attention_tc_long(tm_q, tm_kv, s->tm_pool, tl, sms, st);
+                               e = launch_attention_tc_long(tm_q, tm_kv, tm_kv64, s->tm_pool, tl, sms, st);
                              }
                              if (e == cudaSuccess && aa.n_items > 0) e = launch_attention(s->tm_pool, aa, st);
                              return e;

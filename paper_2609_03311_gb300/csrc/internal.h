@@ -257,13 +257,14 @@ struct AttnTcArgs {
 // Q rows per head in a 128-row tile; 0 when the group size does not divide 128 into boxes of >= 8 rows.
 inline int attn_tc_rows_per_head(int G) { return (G >= 1 && G <= 16 && 128 % G == 0) ? 128 / G : 0; }
 cudaError_t attn_tc_setup();
-// tm_q: the chunk's packed QKV buffer, box 64 columns x (128 / G) rows; tm_kv: the same
-// buffer, box 64 x 16; tm_pool: the store pool, box 64 x 64 (all fp16, 128-byte swizzle).
-cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool,
-                                const AttnTcArgs& a, int num_sms, cudaStream_t st);
+// tm_q: the chunk's packed QKV buffer, box 64 columns x (128 / G) rows; tm_kv and tm_kv64: the
+// same buffer, boxes 64 x 16 and 64 x 64; tm_pool: the store pool, box 64 x 64 (all fp16, 128-byte
+// swizzle).
+cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv64,
+                                const CUtensorMap& tm_pool, const AttnTcArgs& a, int num_sms, cudaStream_t st);
 // Tiles with more than ATTN_TC_MAX_KEYS key columns (same maps and arguments).
-cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool,
-                                     const AttnTcArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv64,
+                                     const CUtensorMap& tm_pool, const AttnTcArgs& a, int num_sms, cudaStream_t st);
 
 // Packer.
 struct PackArgs {

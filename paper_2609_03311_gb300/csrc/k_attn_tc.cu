@@ -167,7 +167,8 @@ __device__ __forceinline__ float exp_pack(uint32_t (&v)[32], uint32_t mask, floa
 
 __global__ void __launch_bounds__(THREADS, 1)
     k_attn_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
-              const __grid_constant__ CUtensorMap tm_pool, AttnTcArgs a) {
+              const __grid_constant__ CUtensorMap tm_kv64, const __grid_constant__ CUtensorMap tm_pool,
+              AttnTcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t s0 = smem_u32(smem);
@@ -205,6 +206,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     fence_mbar_init();
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_kv);
+    tma_prefetch_desc(&tm_kv64);
     tma_prefetch_desc(&tm_pool);
   }
   if (warp == 1) {
@@ -259,16 +261,29 @@ __global__ void __launch_bounds__(THREADS, 1)
           } else {
             const int groups = min(KBLK, n_keys - j * KBLK) / GROUP_ROWS;
             arm(full0 + r.stage, r.phase, groups * GROUP_BYTES);
-            for (int q = 0; q < groups; ++q) {
-              const int off = key - j * KBLK;  // 0, 16, 32, 48 when the plan is consistent
-              if (off >= 0 && off < KBLK)      // otherwise the copy is skipped and the wait times out
-                for (int h = 0; h < 2; ++h)
-                  tma_load_2d(dst + off * 128 + h * KV_HALF, &tm_kv, fb, col0 + h * 64, tok_begin + seg_start(sv) + k);
-              key += GROUP_ROWS;
-              k += GROUP_ROWS;
+            if (groups * GROUP_ROWS == KBLK && key == j * KBLK && k + KBLK <= seg_len(sv)) {
+              // the whole block is 64 consecutive tokens of one pair: one 64-row box per half
+              for (int h = 0; h < 2; ++h)
+                tma_load_2d(dst + h * KV_HALF, &tm_kv64, fb, col0 + h * 64, tok_begin + seg_start(sv) + k);
+              key += KBLK;
+              k += KBLK;
               if (k >= seg_len(sv) && si + 1 < ATTN_TC_MAX_SEGS) {
                 k = 0;
                 sv = tp->seg[++si];
+              }
+            } else {
+              for (int q = 0; q < groups; ++q) {
+                const int off = key - j * KBLK;  // 0, 16, 32, 48 when the plan is consistent
+                if (off >= 0 && off < KBLK)      // otherwise the copy is skipped and the wait times out
+                  for (int h = 0; h < 2; ++h)
+                    tma_load_2d(dst + off * 128 + h * KV_HALF, &tm_kv, fb, col0 + h * 64,
+                                tok_begin + seg_start(sv) + k);
+                key += GROUP_ROWS;
+                k += GROUP_ROWS;
+                if (k >= seg_len(sv) && si + 1 < ATTN_TC_MAX_SEGS) {
+                  k = 0;
+                  sv = tp->seg[++si];
+                }
               }
             }
           }
@@ -555,7 +570,8 @@ static_assert(P_COL + 32 * P_STAGES <= TMEM_COLS, "P ring inside the allocation"
 
 __global__ void __launch_bounds__(lt::THREADS, 1)
     k_attn_tc_long(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
-                   const __grid_constant__ CUtensorMap tm_pool, AttnTcArgs a) {
+                   const __grid_constant__ CUtensorMap tm_kv64, const __grid_constant__ CUtensorMap tm_pool,
+                   AttnTcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t s0 = smem_u32(smem);
@@ -597,6 +613,7 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
     fence_mbar_init();
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_kv);
+    tma_prefetch_desc(&tm_kv64);
     tma_prefetch_desc(&tm_pool);
   }
   if (warp == 1) {
@@ -645,14 +662,25 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
         } else {
           const int groups = min(KBLK, tp->n_keys - j * KBLK) / GROUP_ROWS;
           arm(full0 + r.stage, r.phase, groups * GROUP_BYTES);
-          for (int q = 0; q < groups; ++q) {
+          if (groups * GROUP_ROWS == KBLK && st.k + KBLK <= seg_len(st.sv)) {
+            // the whole block is 64 consecutive tokens of one pair: one 64-row box per half
             for (int h = 0; h < 2; ++h)
-              tma_load_2d(dst + q * GROUP_ROWS * 128 + h * KV_HALF, &tm_kv, fb, st.col0 + h * 64,
-                          tp->tok_begin + seg_start(st.sv) + st.k);
-            st.k += GROUP_ROWS;
+              tma_load_2d(dst + h * KV_HALF, &tm_kv64, fb, st.col0 + h * 64, tp->tok_begin + seg_start(st.sv) + st.k);
+            st.k += KBLK;
             if (st.k >= seg_len(st.sv) && st.si + 1 < ATTN_TC_MAX_SEGS) {
               st.k = 0;
               st.sv = tp->seg[++st.si];
+            }
+          } else {
+            for (int q = 0; q < groups; ++q) {
+              for (int h = 0; h < 2; ++h)
+                tma_load_2d(dst + q * GROUP_ROWS * 128 + h * KV_HALF, &tm_kv, fb, st.col0 + h * 64,
+                            tp->tok_begin + seg_start(st.sv) + st.k);
+              st.k += GROUP_ROWS;
+              if (st.k >= seg_len(st.sv) && st.si + 1 < ATTN_TC_MAX_SEGS) {
+                st.k = 0;
+                st.sv = tp->seg[++st.si];
+              }
             }
           }
         }
@@ -914,19 +942,19 @@ cudaError_t attn_tc_setup() {
   return cudaFuncSetAttribute(k_attn_tc_long, cudaFuncAttributeMaxDynamicSharedMemorySize, lt::SMEM_BYTES);
 }
 
-cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool,
-                                const AttnTcArgs& a, int num_sms, cudaStream_t st) {
+cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv64,
+                                const CUtensorMap& tm_pool, const AttnTcArgs& a, int num_sms, cudaStream_t st) {
   if (a.n_units <= 0) return cudaSuccess;
   const int grid = a.n_units < num_sms ? a.n_units : num_sms;
-  k_attn_tc<<<grid, THREADS, SMEM_BYTES, st>>>(tm_q, tm_kv, tm_pool, a);
+  k_attn_tc<<<grid, THREADS, SMEM_BYTES, st>>>(tm_q, tm_kv, tm_kv64, tm_pool, a);
   return cudaGetLastError();
 }
 
-cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool,
-                                     const AttnTcArgs& a, int num_sms, cudaStream_t st) {
+cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv64,
+                                     const CUtensorMap& tm_pool, const AttnTcArgs& a, int num_sms, cudaStream_t st) {
   if (a.n_units <= 0) return cudaSuccess;
   const int grid = a.n_units < num_sms ? a.n_units : num_sms;
-  k_attn_tc_long<<<grid, lt::THREADS, lt::SMEM_BYTES, st>>>(tm_q, tm_kv, tm_pool, a);
+  k_attn_tc_long<<<grid, lt::THREADS, lt::SMEM_BYTES, st>>>(tm_q, tm_kv, tm_kv64, tm_pool, a);
   return cudaGetLastError();
 }
 
