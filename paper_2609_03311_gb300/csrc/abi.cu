@@ -583,14 +583,15 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     const double attn_bytes_last = np * 2.0 * Hq * HEAD_DIM * 2 + T * 2.0 * Hkv * HEAD_DIM * 2 +
                                    prefix_rows * Hkv * 2 * HEAD_DIM * 2;
     // this chunk's packed QKV buffer as TMA maps for the tensor-core attention:
-    // Q boxes of 128 / G rows per q head, own-key boxes of 16 and of 64 rows
+    // Q boxes of 128 / G rows of the group's G heads, own-key boxes of 16, 32 and 64 rows
     const int TT = attn_tc_rows_per_head(Hq / Hkv);
-    CUtensorMap tm_q{}, tm_kv{}, tm_kv64{};
+    CUtensorMap tm_q{}, tm_kv{}, tm_kv32{}, tm_kv64{};
     const int n_tiles = plan.chunk_tile[ci + 1] - plan.chunk_tile[ci];
     const int n_ltiles = plan.chunk_ltile[ci + 1] - plan.chunk_ltile[ci];
     if (n_tiles + n_ltiles > 0 &&
-        !(make_tmap_16b_2d(&tm_q, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, TT, true, true) &&
+        !(make_tmap_q_heads(&tm_q, w.qkv, m->qkv_dim, Tc, TT, Hq / Hkv) &&
           make_tmap_16b_2d(&tm_kv, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, 16, true, true) &&
+          make_tmap_16b_2d(&tm_kv32, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, 32, true, true) &&
           make_tmap_16b_2d(&tm_kv64, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, 64, true, true)))
       return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for the QKV buffer");
     AttnTcArgs ta{};
@@ -698,11 +699,11 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
                              cudaError_t e = cudaSuccess;
                              if (!last && ta.n_units > 0) {
                                ta.layer = l;
-                               e = launch_attention_tc(tm_q, tm_kv, tm_kv64, s->tm_pool, ta, sms, st);
+                               e = launch_attention_tc(tm_q, tm_kv, tm_kv32, tm_kv64, s->tm_pool, ta, sms, st);
                              }
                              if (e == cudaSuccess && !last && tl.n_units > 0) {
                                tl.layer = l;
-                               e = launch_attention_tc_long(tm_q, tm_kv, tm_kv64, s->tm_pool, tl, sms, st);
+                               e = launch_attention_tc_long(tm_q, tm_kv, tm_kv32, tm_kv64, s->tm_pool, tl, sms, st);
                              }
                              if (e == cudaSuccess && aa.n_items > 0) e = launch_attention(s->tm_pool, aa, st);
                              return e;
@@ -863,6 +864,23 @@ bool make_tmap_16b_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_
                   CU_TENSOR_MAP_INTERLEAVE_NONE,
                   swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// The Q columns of a packed QKV buffer [rows][cols] as a 3-D tensor: 128 elements of a head
+// (innermost), rows, heads (256 bytes apart); the box takes 64 elements of box_heads heads over
+// box_rows rows, stored head after head (fp16, 128-byte swizzle).
+bool make_tmap_q_heads(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows,
+                       uint32_t box_heads) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {128, rows, cols / 128};
+  cuuint64_t strides[2] = {cols * 2, 256};
+  cuuint32_t box[3] = {64, box_rows, box_heads};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
 

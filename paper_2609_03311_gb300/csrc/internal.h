@@ -164,6 +164,8 @@ struct Model {
 // 2-D map over 16-bit elements (fp16 when `half` is set, else bf16).
 bool make_tmap_16b_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
                       uint32_t box_cols, uint32_t box_rows, bool swizzle128, bool half);
+bool make_tmap_q_heads(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows,
+                       uint32_t box_heads);
 
 // GEMM epilogues.
 enum GemmEpi : int { EPI_STORE = 0, EPI_RESID_ADD = 1, EPI_SWIGLU = 2, EPI_QKV = 3 };
@@ -257,14 +259,16 @@ struct AttnTcArgs {
 // Q rows per head in a 128-row tile; 0 when the group size does not divide 128 into boxes of >= 8 rows.
 inline int attn_tc_rows_per_head(int G) { return (G >= 1 && G <= 16 && 128 % G == 0) ? 128 / G : 0; }
 cudaError_t attn_tc_setup();
-// tm_q: the chunk's packed QKV buffer, box 64 columns x (128 / G) rows; tm_kv and tm_kv64: the
-// same buffer, boxes 64 x 16 and 64 x 64; tm_pool: the store pool, box 64 x 64 (all fp16, 128-byte
-// swizzle).
-cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv64,
-                                const CUtensorMap& tm_pool, const AttnTcArgs& a, int num_sms, cudaStream_t st);
+// tm_q: the Q heads of the chunk's packed QKV buffer as a 3-D map (make_tmap_q_heads), box 64
+// columns x (128 / G) rows x G heads; tm_kv, tm_kv32, tm_kv64: the same buffer, boxes 64 x 16,
+// 64 x 32 and 64 x 64; tm_pool: the store pool, box 64 x 64 (all fp16, 128-byte swizzle).
+cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv32,
+                                const CUtensorMap& tm_kv64, const CUtensorMap& tm_pool, const AttnTcArgs& a,
+                                int num_sms, cudaStream_t st);
 // Tiles with more than ATTN_TC_MAX_KEYS key columns (same maps and arguments).
-cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv64,
-                                     const CUtensorMap& tm_pool, const AttnTcArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv32,
+                                     const CUtensorMap& tm_kv64, const CUtensorMap& tm_pool, const AttnTcArgs& a,
+                                     int num_sms, cudaStream_t st);
 
 // Packer.
 struct PackArgs {

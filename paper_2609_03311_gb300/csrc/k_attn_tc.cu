@@ -167,8 +167,8 @@ __device__ __forceinline__ float exp_pack(uint32_t (&v)[32], uint32_t mask, floa
 
 __global__ void __launch_bounds__(THREADS, 1)
     k_attn_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
-              const __grid_constant__ CUtensorMap tm_kv64, const __grid_constant__ CUtensorMap tm_pool,
-              AttnTcArgs a) {
+              const __grid_constant__ CUtensorMap tm_kv32, const __grid_constant__ CUtensorMap tm_kv64,
+              const __grid_constant__ CUtensorMap tm_pool, AttnTcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t s0 = smem_u32(smem);
@@ -206,6 +206,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     fence_mbar_init();
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_kv);
+    tma_prefetch_desc(&tm_kv32);
     tma_prefetch_desc(&tm_kv64);
     tma_prefetch_desc(&tm_pool);
   }
@@ -233,10 +234,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       auto issue_q = [&](int tok_begin, int g) -> bool {
         if (!mbar_wait(bar(BAR_Q_EMPTY + rq.stage), rq.phase ^ 1u, a.err, WAIT_TIMEOUT_NS)) return false;
         arm(BAR_Q_FULL + rq.stage, rq.phase, Q_BYTES);
-        for (int hh = 0; hh < G; ++hh)  // one box of TT rows per (q head of the group, 64-column half)
-          for (int h = 0; h < 2; ++h)
-            tma_load_2d(sQ + rq.stage * Q_BYTES + h * Q_HALF + hh * TT * 128, &tm_q, bar(BAR_Q_FULL + rq.stage),
-                        (g * G + hh) * HEAD_DIM + h * 64, tok_begin);
+        for (int h = 0; h < 2; ++h)  // one box per 64-column half: TT rows of each of the group's G heads
+          tma_load_3d(sQ + rq.stage * Q_BYTES + h * Q_HALF, &tm_q, bar(BAR_Q_FULL + rq.stage), h * 64, tok_begin,
+                      g * G);
         rq.next(Q_STAGES);
         return true;
       };
@@ -272,14 +272,17 @@ __global__ void __launch_bounds__(THREADS, 1)
                 sv = tp->seg[++si];
               }
             } else {
-              for (int q = 0; q < groups; ++q) {
+              for (int q = 0; q < groups;) {
                 const int off = key - j * KBLK;  // 0, 16, 32, 48 when the plan is consistent
-                if (off >= 0 && off < KBLK)      // otherwise the copy is skipped and the wait times out
+                // two groups at once when both are 16 consecutive visible tokens of this pair
+                const int n = (q + 2 <= groups && k + 2 * GROUP_ROWS <= seg_len(sv)) ? 2 : 1;
+                if (off >= 0 && off + n * GROUP_ROWS <= KBLK)  // otherwise skipped and the wait times out
                   for (int h = 0; h < 2; ++h)
-                    tma_load_2d(dst + off * 128 + h * KV_HALF, &tm_kv, fb, col0 + h * 64,
+                    tma_load_2d(dst + off * 128 + h * KV_HALF, n == 2 ? &tm_kv32 : &tm_kv, fb, col0 + h * 64,
                                 tok_begin + seg_start(sv) + k);
-                key += GROUP_ROWS;
-                k += GROUP_ROWS;
+                key += n * GROUP_ROWS;
+                k += n * GROUP_ROWS;
+                q += n;
                 if (k >= seg_len(sv) && si + 1 < ATTN_TC_MAX_SEGS) {
                   k = 0;
                   sv = tp->seg[++si];
@@ -570,8 +573,8 @@ static_assert(P_COL + 32 * P_STAGES <= TMEM_COLS, "P ring inside the allocation"
 
 __global__ void __launch_bounds__(lt::THREADS, 1)
     k_attn_tc_long(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
-                   const __grid_constant__ CUtensorMap tm_kv64, const __grid_constant__ CUtensorMap tm_pool,
-                   AttnTcArgs a) {
+                   const __grid_constant__ CUtensorMap tm_kv32, const __grid_constant__ CUtensorMap tm_kv64,
+                   const __grid_constant__ CUtensorMap tm_pool, AttnTcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t s0 = smem_u32(smem);
@@ -613,6 +616,7 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
     fence_mbar_init();
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_kv);
+    tma_prefetch_desc(&tm_kv32);
     tma_prefetch_desc(&tm_kv64);
     tma_prefetch_desc(&tm_pool);
   }
@@ -672,11 +676,14 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
               st.sv = tp->seg[++st.si];
             }
           } else {
-            for (int q = 0; q < groups; ++q) {
+            for (int q = 0; q < groups;) {
+              // two groups at once when both are 16 consecutive visible tokens of this pair
+              const int n = (q + 2 <= groups && st.k + 2 * GROUP_ROWS <= seg_len(st.sv)) ? 2 : 1;
               for (int h = 0; h < 2; ++h)
-                tma_load_2d(dst + q * GROUP_ROWS * 128 + h * KV_HALF, &tm_kv, fb, st.col0 + h * 64,
-                            tp->tok_begin + seg_start(st.sv) + st.k);
-              st.k += GROUP_ROWS;
+                tma_load_2d(dst + q * GROUP_ROWS * 128 + h * KV_HALF, n == 2 ? &tm_kv32 : &tm_kv, fb,
+                            st.col0 + h * 64, tp->tok_begin + seg_start(st.sv) + st.k);
+              st.k += n * GROUP_ROWS;
+              q += n;
               if (st.k >= seg_len(st.sv) && st.si + 1 < ATTN_TC_MAX_SEGS) {
                 st.k = 0;
                 st.sv = tp->seg[++st.si];
@@ -699,10 +706,9 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
           break;
         }
         arm(lt::B_Q_FULL + rq.stage, rq.phase, Q_BYTES);
-        for (int hh = 0; hh < G; ++hh)
-          for (int h = 0; h < 2; ++h)
-            tma_load_2d(sQ + rq.stage * Q_BYTES + h * Q_HALF + hh * TT * 128, &tm_q, bar(lt::B_Q_FULL + rq.stage),
-                        (g * G + hh) * HEAD_DIM + h * 64, tp->tok_begin);
+        for (int h = 0; h < 2; ++h)
+          tma_load_3d(sQ + rq.stage * Q_BYTES + h * Q_HALF, &tm_q, bar(lt::B_Q_FULL + rq.stage), h * 64,
+                      tp->tok_begin, g * G);
         rq.next(lt::Q_STAGES);
         Stream ka = start(tp, g, 0);
         for (int j = 0; j < nb && ok; ++j) ok = issue_block(tp, ka, j);
@@ -942,19 +948,21 @@ cudaError_t attn_tc_setup() {
   return cudaFuncSetAttribute(k_attn_tc_long, cudaFuncAttributeMaxDynamicSharedMemorySize, lt::SMEM_BYTES);
 }
 
-cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv64,
-                                const CUtensorMap& tm_pool, const AttnTcArgs& a, int num_sms, cudaStream_t st) {
+cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv32,
+                                const CUtensorMap& tm_kv64, const CUtensorMap& tm_pool, const AttnTcArgs& a,
+                                int num_sms, cudaStream_t st) {
   if (a.n_units <= 0) return cudaSuccess;
   const int grid = a.n_units < num_sms ? a.n_units : num_sms;
-  k_attn_tc<<<grid, THREADS, SMEM_BYTES, st>>>(tm_q, tm_kv, tm_kv64, tm_pool, a);
+  k_attn_tc<<<grid, THREADS, SMEM_BYTES, st>>>(tm_q, tm_kv, tm_kv32, tm_kv64, tm_pool, a);
   return cudaGetLastError();
 }
 
-cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv64,
-                                     const CUtensorMap& tm_pool, const AttnTcArgs& a, int num_sms, cudaStream_t st) {
+cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv32,
+                                     const CUtensorMap& tm_kv64, const CUtensorMap& tm_pool, const AttnTcArgs& a,
+                                     int num_sms, cudaStream_t st) {
   if (a.n_units <= 0) return cudaSuccess;
   const int grid = a.n_units < num_sms ? a.n_units : num_sms;
-  k_attn_tc_long<<<grid, lt::THREADS, lt::SMEM_BYTES, st>>>(tm_q, tm_kv, tm_kv64, tm_pool, a);
+  k_attn_tc_long<<<grid, lt::THREADS, lt::SMEM_BYTES, st>>>(tm_q, tm_kv, tm_kv32, tm_kv64, tm_pool, a);
   return cudaGetLastError();
 }
 
