@@ -51,3 +51,29 @@ def test_full_size_batch_matches_oracle_on_sampled_pairs(workload, n_oracle):
         np.testing.assert_array_equal(got2, got[rev])
     model.close()
     store.close()
+
+
+def test_full_size_candidate_list_ranking_matches_oracle():
+    # One query's complete candidate list at the full Qwen3-0.6B size (28 layers), scored inside
+    # the bench's batch: every score within 3e-2 of the oracle, and the top-10 order identical
+    # wherever the oracle's adjacent gap exceeds 0.1.
+    wl = synth.WORKLOADS["qwen3-0.6b"]
+    dev = torch.device("cuda")
+    cfg, model, store, doc_m, w_host = bench.setup(wl, 0, dev, need_host_weights=True)
+    pairs = bench.build_pairs(wl, 0)
+    per_q = wl.docs_per_query
+    b = bench.slice_pairs(pairs, 0, 20 * per_q)
+    got = dopr.score(model, store, torch.tensor(b["q_offsets"], device=dev), torch.tensor(b["q_tokens"], device=dev),
+                     torch.tensor(b["doc_ids"], device=dev)).cpu().numpy()
+    idx = list(range(per_q))  # the first query's candidates
+    assert len(set(np.diff(pairs["q_offsets"])[idx])) == 1  # one query: the same length throughout
+    ref_d, _, _ = bench.oracle_sample(wl, w_host, doc_m, pairs, idx, 0, 1e9, dev)
+    ref = np.array([ref_d[p] for p in idx])
+    g = got[:per_q]
+    assert np.max(np.abs(g - ref)) <= TOL, float(np.max(np.abs(g - ref)))
+    order = np.argsort(-ref, kind="stable")[:10]
+    for a, c in zip(order[:-1], order[1:]):
+        if ref[a] - ref[c] > 0.1:
+            assert g[a] > g[c], (int(a), int(c))
+    model.close()
+    store.close()
