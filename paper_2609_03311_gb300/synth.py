@@ -78,6 +78,7 @@ class Workload:
     qlen_max: int
     zipf_s: float = 0.0         # 0 -> uniform candidate draw
     fulldoc_tokens: int = 0     # >0: the uncompressed comparison run
+    pair_set: str = ""          # workloads naming the same pair set score the same pairs (default: own name)
 
     @property
     def n_pairs(self) -> int:
@@ -92,11 +93,13 @@ WORKLOADS = {
     # Qwen3-4B, 2000 docs m=128, 50 x 200 pairs, queries 32..256 tokens.
     "qwen3-4b": Workload("qwen3-4b", MODELS["qwen3-4b"], 2000, (128,), 50, 200, 32, 256),
     # Qwen3-8B, 1000 docs m in {32,64,128,256}, 200 x 100 Zipf(1.1) pairs, queries 8..64.
-    "qwen3-8b-zipf": Workload("qwen3-8b-zipf", MODELS["qwen3-8b"], 1000, (32, 64, 128, 256), 200, 100, 8, 64, 1.1),
-    # Same pairs as above with every prefix m=64 (the headline workload).
+    "qwen3-8b-zipf": Workload("qwen3-8b-zipf", MODELS["qwen3-8b"], 1000, (32, 64, 128, 256), 200, 100, 8, 64, 1.1,
+                              pair_set="qwen3-8b-m64"),
+    # The same pairs with every prefix m=64 (the headline workload).
     "qwen3-8b-m64": Workload("qwen3-8b-m64", MODELS["qwen3-8b"], 1000, (64,), 200, 100, 8, 64, 1.1),
-    # Uncompressed comparison: [512 doc tokens ; query ; score token], no prefix.
-    "qwen3-8b-fulldoc": Workload("qwen3-8b-fulldoc", MODELS["qwen3-8b"], 1000, (0,), 200, 100, 8, 64, 1.1, 512),
+    # The same pairs scored uncompressed: [512 doc tokens ; query ; score token], no prefix.
+    "qwen3-8b-fulldoc": Workload("qwen3-8b-fulldoc", MODELS["qwen3-8b"], 1000, (0,), 200, 100, 8, 64, 1.1, 512,
+                                 pair_set="qwen3-8b-m64"),
 }
 
 
@@ -213,7 +216,7 @@ def make_workload_pairs(wl: Workload, seed: int = 0):
     """Pair list of a workload.  Returns dict with q_offsets [n+1] int32,
     q_tokens int32, doc_ids [n] int64, query_of_pair [n] int32 (pairs are
     listed query by query, each query's candidates in draw order)."""
-    rng = np.random.default_rng(sub_seed(seed, "pairs", wl.name))
+    rng = np.random.default_rng(sub_seed(seed, "pairs", wl.pair_set or wl.name))
     n_docs, k = wl.n_docs, wl.docs_per_query
     if wl.zipf_s > 0:
         order = rng.permutation(n_docs)            # rank -> doc id
