@@ -38,13 +38,22 @@ sys.path.insert(0, ROOT)
 METRIC = "scored query-doc pairs/sec at 1 GB300 (Qwen3-8B shape, m=64); p50 batch latency"
 
 
-def parse_args():
+# The workloads of the five measured configurations, by number: 0 the 2-layer Qwen3-0.6B-width
+# case, 1 Qwen3-0.6B, 2 Qwen3-4B with long queries, 3 Qwen3-8B with Zipf reuse and mixed prefix
+# lengths, 4 the uncompressed comparison of config 3's pairs; "3'" (m = 64 throughout) is the headline.
+CONFIG_WORKLOADS = {"0": "qwen3-0.6b-2l", "1": "qwen3-0.6b", "2": "qwen3-4b", "3": "qwen3-8b-zipf",
+                    "3'": "qwen3-8b-m64", "4": "qwen3-8b-fulldoc"}
+
+
+def parse_args(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["dopr", "reference"], default="dopr")
     ap.add_argument("--workload", default="qwen3-8b-m64")
+    ap.add_argument("--config", choices=sorted(CONFIG_WORKLOADS), default=None,
+                    help="select the workload by configuration number (overrides --workload)")
     ap.add_argument("--queries-per-step", type=int, default=20)
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="bound of the oracle CPU-baseline sample")
@@ -53,7 +62,10 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--reuse", action="store_true",
                     help="amortised cost under document reuse (T_off, T_full, T_online, Speedup(r)) instead of the bench")
-    return ap.parse_args()
+    args = ap.parse_args(argv)
+    if args.config is not None:
+        args.workload = CONFIG_WORKLOADS[args.config]
+    return args
 
 
 def measured_peaks():

@@ -76,3 +76,12 @@ def test_reference_arm_under_two_ranks_prints_one_line():
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
     assert d["cpu_baseline"]["kind"] == "oracle" and d["e2e"]["h2d_bytes_per_step"] == 0
+
+
+def test_config_numbers_select_the_workloads():
+    from paper_2609_03311_gb300 import synth
+
+    assert set(bench.CONFIG_WORKLOADS.values()) == set(synth.WORKLOADS)
+    assert bench.parse_args(["--config", "3'"]).workload == "qwen3-8b-m64"
+    assert bench.parse_args(["--config", "2"]).workload == "qwen3-4b"
+    assert bench.parse_args([]).workload == "qwen3-8b-m64"  # the headline by default
