@@ -19,6 +19,8 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include <algorithm>
 #include <memory>
 #include <mutex>
@@ -32,6 +34,20 @@ struct dopr_model : dopr::Model {};
 struct dopr_store : dopr::Store {};
 
 namespace dopr {
+
+// A named NVTX range for the lifetime of the object (per call, chunk and layer), so a
+// profiler can attribute kernels; it costs a function call when no tool is attached.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  NvtxRange(const char* fmt, int v) {
+    char b[48];
+    snprintf(b, sizeof b, fmt, v);
+    nvtxRangePushA(b);
+  }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 namespace {
 
 thread_local std::string g_last_error;
@@ -548,6 +564,7 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     return std::make_pair(2.0 * M * N * K, (M * K + N * K) * 2.0 + out_bytes);
   };
   for (size_t ci = 0; ci + 1 < plan.chunk_pair.size(); ++ci) {
+    NvtxRange chunk_range("dopr chunk %d", static_cast<int>(ci));
     const int32_t s0 = plan.chunk_pair[ci], s1 = plan.chunk_pair[ci + 1];
     const int32_t t0 = w.h_tok_off[s0], Tc = w.h_tok_off[s1] - t0;
     const double T = Tc;
@@ -611,6 +628,7 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     const auto gu_last = gemm_cost(np, 2.0 * F, H, np * F * 2.0);
     const auto dn_last = gemm_cost(np, H, F, np * H * 8.0);
     for (int l = 0; l < L; ++l) {
+      NvtxRange layer_range("dopr layer %d", l);
       // In the last layer only the score-token rows reach the score: after the full QKV
       // projection (every token's key and value is attended to), attention, O and the MLP
       // run on one compact row per pair.
@@ -1145,6 +1163,7 @@ dopr_status dopr_store_put(dopr_store* s, int64_t doc_id, int32_t m, int32_t lay
 dopr_status dopr_build_prefixes(dopr_model* m, dopr_store* s, int32_t n_docs, const int64_t* doc_ids,
                                 const int32_t* x_offsets, const void* x, int32_t x_on_device, void* cuda_stream) {
   g_last_error.clear();
+  NvtxRange call_range("dopr_build_prefixes");
   STATUS_TRY(check_ready(m, s));
   if (n_docs < 0) return fail(DOPR_ERR_INVALID_ARG, "n_docs < 0");
   if (n_docs == 0) return DOPR_OK;
@@ -1251,6 +1270,7 @@ dopr_status dopr_select_prefix_inputs(dopr_model* m, int32_t n_docs, const int32
                                       const int32_t* doc_tokens, int32_t top_k, int32_t top_p, int32_t* positions,
                                       void* x_out, float* salience, void* cuda_stream) {
   g_last_error.clear();
+  NvtxRange call_range("dopr_select_prefix_inputs");
   if (!m) return fail(DOPR_ERR_INVALID_ARG, "model is NULL");
   const auto& c = m->cfg;
   const int H = c.hidden, L = c.n_layers;
@@ -1389,6 +1409,7 @@ dopr_status dopr_store_destroy(dopr_store* s) {
 dopr_status dopr_score(dopr_model* m, dopr_store* s, int32_t n, const int32_t* q_offsets, const int32_t* q_tokens,
                        const int64_t* doc_ids, float* scores, void* cuda_stream, int32_t io_on_device) {
   g_last_error.clear();
+  NvtxRange call_range("dopr_score");
   STATUS_TRY(check_ready(m, s));
   if (n < 0) return fail(DOPR_ERR_INVALID_ARG, "n_pairs < 0");
   if (n == 0) return DOPR_OK;
