@@ -38,9 +38,9 @@ sys.path.insert(0, ROOT)
 METRIC = "scored query-doc pairs/sec at 1 GB300 (Qwen3-8B shape, m=64); p50 batch latency"
 
 
-# The workloads of the five measured configurations, by number: 0 the 2-layer Qwen3-0.6B-width
-# case, 1 Qwen3-0.6B, 2 Qwen3-4B with long queries, 3 Qwen3-8B with Zipf reuse and mixed prefix
-# lengths, 4 the uncompressed comparison of config 3's pairs; "3'" (m = 64 throughout) is the headline.
+# Short numbers for the measured workloads: 0 the 2-layer Qwen3-0.6B-width case, 1 Qwen3-0.6B,
+# 2 Qwen3-4B with long queries, 3 Qwen3-8B with Zipf reuse and mixed prefix lengths, 3' the same
+# Qwen3-8B pairs with m = 64 throughout (the default), 4 those pairs scored uncompressed.
 CONFIG_WORKLOADS = {"0": "qwen3-0.6b-2l", "1": "qwen3-0.6b", "2": "qwen3-4b", "3": "qwen3-8b-zipf",
                     "3'": "qwen3-8b-m64", "4": "qwen3-8b-fulldoc"}
 
@@ -427,7 +427,7 @@ def run_dopr(args, rank, world, local_rank, dist):
             "vs_baseline": None, "dtype": "f16",
             "data": "synthetic: seeded random-init bf16 weights N(0,0.02), N(0,1) prefix K/V, uniform token ids",
             "config": {"workload": wl.name,
-                       "model": f"{wl.model.name}: {wl.model.n_layers} layers, hidden {wl.model.hidden}, "
+                       "decoder": f"{wl.model.name}: {wl.model.n_layers} layers, hidden {wl.model.hidden}, "
                                 f"{wl.model.n_q_heads}/{wl.model.n_kv_heads} heads, head_dim 128, ffn {wl.model.ffn}",
                        "docs": wl.n_docs, "m": list(wl.m_choices), "fulldoc_tokens": wl.fulldoc_tokens,
                        "pairs_per_step": Q * per_q, "queries_per_step": Q, "query_len": [wl.qlen_min, wl.qlen_max],
@@ -522,7 +522,7 @@ def run_reuse(args):
     rs = [1, 2, 4, 8, 16, 32, 64, 128]
     print(json.dumps({
         "metric": "amortised speedup under document reuse, r T_full / (T_off + r T_online)", "unit": "x",
-        "config": {"workload": wl.name, "model": s.name, "m": m, "document_tokens": n_doc_tokens,
+        "config": {"workload": wl.name, "decoder": s.name, "m": m, "document_tokens": n_doc_tokens,
                    "online_pairs": n_on, "full_pairs": n_full, "offline_documents": len(docs)},
         "t_online_ms_per_pair": t_online, "t_full_ms_per_pair": t_full,
         "t_off_ms_per_doc": t_off, "t_off_parts_ms": {"key_token_selection": t_doc, "prefix_build": t_build},
