@@ -18,9 +18,11 @@
 //   warp 0    TMA producer: the Q tile (two stages), the tile's key blocks of
 //             64 columns into a K ring (five stages) and a V ring (three) --
 //             prefix blocks from the store pool in 64-row boxes, own-key
-//             segments from the packed QKV buffer in 16-row boxes;
-//   warp 1    MMA issuer: S = Q K^T for every key block into the unit's TMEM
-//             region (fp32, up to 256 columns), then O = P V block by block
+//             segments from the packed QKV buffer in the largest of 64-, 32-
+//             or 16-row boxes that stays inside one pair's visible tokens;
+//   warp 1    MMA issuer: S = Q K^T into the unit's TMEM region (fp32, up to
+//             256 columns; one MMA per 16-element step spans every key block
+//             held in consecutive ring stages), then O = P V block by block
 //             with P read from TMEM and V from shared memory as an MN-major
 //             operand, into the region's upper 128 columns (over S blocks 2
 //             and 3, when the unit has them, once the softmax has read them);
@@ -62,6 +64,10 @@ constexpr int MAX_BLOCKS = ATTN_TC_MAX_KEYS / KBLK;  // 4
 // S blocks 2 and 3 when the unit has them.
 constexpr uint32_t TMEM_COLS = 512, SLOT_COLS = 256, O_COL = 128;
 
+// Shared memory.  The K ring is half-major ([half][stage][64 rows][128 B]): the
+// rows of consecutive stages follow one another, so the blocks of a unit that
+// sit in consecutive stages are one K-major operand for a single wide S MMA.
+// Q and V stages keep their two 64-column halves together.
 constexpr int OFF_Q = 0;
 constexpr int OFF_K = OFF_Q + Q_STAGES * Q_BYTES;
 constexpr int OFF_V = OFF_K + K_STAGES * KV_BYTES;
@@ -79,7 +85,6 @@ static_assert(BAR_V_FULL + V_STAGES <= 32, "the producer tracks the barriers it 
 constexpr int SMEM_BYTES = 1024 + OFF_BAR + N_BARS * 8 + 16;
 static_assert(SMEM_BYTES <= 227 * 1024, "shared memory budget");
 
-constexpr uint32_t IDESC_S = umma_idesc_f16(TILE_M, KBLK);
 constexpr uint32_t IDESC_O = umma_idesc_f16_bmn(TILE_M, HEAD_DIM);
 
 struct Ring {
@@ -253,18 +258,20 @@ __global__ void __launch_bounds__(THREADS, 1)
         int sv = tp->seg[0];
         for (int j = 0; j < nb; ++j) {
           if (!mbar_wait(bar(empty0 + r.stage), r.phase ^ 1u, a.err, WAIT_TIMEOUT_NS)) return false;
-          const uint32_t dst = ring + r.stage * KV_BYTES;
+          // half h of the stage: K halves lie K_STAGES * 8 KB apart (see OFF_K), V halves 8 KB apart
+          const uint32_t dst = kv ? ring + r.stage * KV_BYTES : ring + r.stage * KV_HALF;
+          const uint32_t hstride = kv ? KV_HALF : K_STAGES * KV_HALF;
           const uint32_t fb = bar(full0 + r.stage);
           if (j * KBLK < pre64) {
             arm(full0 + r.stage, r.phase, KV_BYTES);
-            for (int h = 0; h < 2; ++h) tma_load_2d(dst + h * KV_HALF, &tm_pool, fb, h * 64, pool_row + j * KBLK);
+            for (int h = 0; h < 2; ++h) tma_load_2d(dst + h * hstride, &tm_pool, fb, h * 64, pool_row + j * KBLK);
           } else {
             const int groups = min(KBLK, n_keys - j * KBLK) / GROUP_ROWS;
             arm(full0 + r.stage, r.phase, groups * GROUP_BYTES);
             if (groups * GROUP_ROWS == KBLK && key == j * KBLK && k + KBLK <= seg_len(sv)) {
               // the whole block is 64 consecutive tokens of one pair: one 64-row box per half
               for (int h = 0; h < 2; ++h)
-                tma_load_2d(dst + h * KV_HALF, &tm_kv64, fb, col0 + h * 64, tok_begin + seg_start(sv) + k);
+                tma_load_2d(dst + h * hstride, &tm_kv64, fb, col0 + h * 64, tok_begin + seg_start(sv) + k);
               key += KBLK;
               k += KBLK;
               if (k >= seg_len(sv) && si + 1 < ATTN_TC_MAX_SEGS) {
@@ -278,7 +285,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const int n = (q + 2 <= groups && k + 2 * GROUP_ROWS <= seg_len(sv)) ? 2 : 1;
                 if (off >= 0 && off + n * GROUP_ROWS <= KBLK)  // otherwise skipped and the wait times out
                   for (int h = 0; h < 2; ++h)
-                    tma_load_2d(dst + off * 128 + h * KV_HALF, n == 2 ? &tm_kv32 : &tm_kv, fb, col0 + h * 64,
+                    tma_load_2d(dst + off * 128 + h * hstride, n == 2 ? &tm_kv32 : &tm_kv, fb, col0 + h * 64,
                                 tok_begin + seg_start(sv) + k);
                 key += n * GROUP_ROWS;
                 k += n * GROUP_ROWS;
@@ -372,17 +379,26 @@ __global__ void __launch_bounds__(THREADS, 1)
             tc_fence_after();
             prog = true;
           }
-          while (s_open && js < nbs && mbar_test(bar(BAR_K_FULL + rk.stage), rk.phase)) {
+          while (s_open && js < nbs) {
+            // the unit's next blocks that sit in consecutive ring stages form one B operand of
+            // 64 * run rows: one N = 64 * run MMA per 16-element step once all of them are in
+            const int run = min(nbs - js, K_STAGES - rk.stage);
+            bool landed = true;
+            for (int t = 0; t < run && landed; ++t) landed = mbar_test(bar(BAR_K_FULL + rk.stage + t), rk.phase);
+            if (!landed) break;
             tc_fence_after();
             const uint64_t qd = umma_desc_sw128(sQ + rq.stage * Q_BYTES);
-            const uint64_t kd = umma_desc_sw128(sK + rk.stage * KV_BYTES);
+            const uint64_t kd = umma_desc_sw128(sK + rk.stage * KV_HALF);
+            const uint32_t idesc = umma_idesc_f16(TILE_M, run * KBLK);
 #pragma unroll
-            for (int ks = 0; ks < HEAD_DIM / 16; ++ks)  // 16 elements = 32 bytes of K per step, halves 16 KB / 8 KB apart
+            for (int ks = 0; ks < HEAD_DIM / 16; ++ks)  // 16 elements = 32 bytes per step; Q halves 16 KB apart
               umma_f16(tmem + slot * SLOT_COLS + js * KBLK, qd + ((ks >> 2) * Q_HALF + (ks & 3) * 32) / 16,
-                       kd + ((ks >> 2) * KV_HALF + (ks & 3) * 32) / 16, IDESC_S, ks > 0);
-            umma_commit(bar(BAR_K_EMPTY + rk.stage));
-            rk.next(K_STAGES);
-            ++js;
+                       kd + ((ks >> 2) * K_STAGES * KV_HALF + (ks & 3) * 32) / 16, idesc, ks > 0);
+            for (int t = 0; t < run; ++t) {
+              umma_commit(bar(BAR_K_EMPTY + rk.stage));
+              rk.next(K_STAGES);
+            }
+            js += run;
             prog = true;
           }
           if (s_open && js == nbs) {
@@ -555,7 +571,7 @@ constexpr int THREADS = 64 + 128;
 // TMEM: O at [0, 128), S buffer b at S_COL + CH b, P stage s (64 keys as fp16) at P_COL + 32 s
 constexpr uint32_t O_COL = 0, S_COL = 128, P_COL = 384;
 constexpr int OFF_Q = 0;
-constexpr int OFF_K = OFF_Q + Q_STAGES * Q_BYTES;
+constexpr int OFF_K = OFF_Q + Q_STAGES * Q_BYTES;  // half-major, as in the short kernel
 constexpr int OFF_V = OFF_K + K_STAGES * KV_BYTES;
 constexpr int OFF_EP = OFF_V + V_STAGES * KV_BYTES;
 constexpr int OFF_BAR = OFF_EP + 4 * EP_WARP_BYTES;
@@ -658,18 +674,20 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
         const int stages = st.kv ? lt::V_STAGES : lt::K_STAGES;
         const int full0 = st.kv ? lt::B_V_FULL : lt::B_K_FULL, empty0 = st.kv ? lt::B_V_EMPTY : lt::B_K_EMPTY;
         if (!mbar_wait(bar(empty0 + r.stage), r.phase ^ 1u, a.err, WAIT_TIMEOUT_NS)) return false;
-        const uint32_t dst = (st.kv ? sV : sK) + r.stage * KV_BYTES;
+        // half h of the stage: K halves lie K_STAGES * 8 KB apart (half-major K ring), V halves 8 KB apart
+        const uint32_t dst = st.kv ? sV + r.stage * KV_BYTES : sK + r.stage * KV_HALF;
+        const uint32_t hstride = st.kv ? KV_HALF : lt::K_STAGES * KV_HALF;
         const uint32_t fb = bar(full0 + r.stage);
         if (j * KBLK < ceil64(tp->m)) {
           arm(full0 + r.stage, r.phase, KV_BYTES);
-          for (int h = 0; h < 2; ++h) tma_load_2d(dst + h * KV_HALF, &tm_pool, fb, h * 64, st.pool_row + j * KBLK);
+          for (int h = 0; h < 2; ++h) tma_load_2d(dst + h * hstride, &tm_pool, fb, h * 64, st.pool_row + j * KBLK);
         } else {
           const int groups = min(KBLK, tp->n_keys - j * KBLK) / GROUP_ROWS;
           arm(full0 + r.stage, r.phase, groups * GROUP_BYTES);
           if (groups * GROUP_ROWS == KBLK && st.k + KBLK <= seg_len(st.sv)) {
             // the whole block is 64 consecutive tokens of one pair: one 64-row box per half
             for (int h = 0; h < 2; ++h)
-              tma_load_2d(dst + h * KV_HALF, &tm_kv64, fb, st.col0 + h * 64, tp->tok_begin + seg_start(st.sv) + st.k);
+              tma_load_2d(dst + h * hstride, &tm_kv64, fb, st.col0 + h * 64, tp->tok_begin + seg_start(st.sv) + st.k);
             st.k += KBLK;
             if (st.k >= seg_len(st.sv) && st.si + 1 < ATTN_TC_MAX_SEGS) {
               st.k = 0;
@@ -680,7 +698,7 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
               // two groups at once when both are 16 consecutive visible tokens of this pair
               const int n = (q + 2 <= groups && st.k + 2 * GROUP_ROWS <= seg_len(st.sv)) ? 2 : 1;
               for (int h = 0; h < 2; ++h)
-                tma_load_2d(dst + q * GROUP_ROWS * 128 + h * KV_HALF, n == 2 ? &tm_kv32 : &tm_kv, fb,
+                tma_load_2d(dst + q * GROUP_ROWS * 128 + h * hstride, n == 2 ? &tm_kv32 : &tm_kv, fb,
                             st.col0 + h * 64, tp->tok_begin + seg_start(st.sv) + st.k);
               st.k += n * GROUP_ROWS;
               q += n;
@@ -736,16 +754,24 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
         if (!wait(lt::B_S_FREE + buf, ((cc >> 1) & 1u) ^ 1u)) return false;
         tc_fence_after();
         const uint64_t qd = umma_desc_sw128(sQ + rq.stage * Q_BYTES);
-        for (int j = 2 * c; j < min(nb, 2 * c + 2); ++j) {
-          if (!wait(lt::B_K_FULL + rk.stage, rk.phase)) return false;
+        const int je = min(nb, 2 * c + 2);
+        for (int j = 2 * c; j < je;) {
+          // the chunk's blocks in consecutive ring stages: one N = 64 * run MMA per step
+          const int run = min(je - j, lt::K_STAGES - rk.stage);
+          for (int t = 0; t < run; ++t)
+            if (!wait(lt::B_K_FULL + rk.stage + t, rk.phase)) return false;
           tc_fence_after();
-          const uint64_t kd = umma_desc_sw128(sK + rk.stage * KV_BYTES);
+          const uint64_t kd = umma_desc_sw128(sK + rk.stage * KV_HALF);
+          const uint32_t idesc = umma_idesc_f16(TILE_M, run * KBLK);
 #pragma unroll
           for (int ks = 0; ks < HEAD_DIM / 16; ++ks)
             umma_f16(tmem + lt::S_COL + lt::CH * buf + (j - 2 * c) * KBLK, qd + ((ks >> 2) * Q_HALF + (ks & 3) * 32) / 16,
-                     kd + ((ks >> 2) * KV_HALF + (ks & 3) * 32) / 16, IDESC_S, ks > 0);
-          umma_commit(bar(lt::B_K_EMPTY + rk.stage));
-          rk.next(lt::K_STAGES);
+                     kd + ((ks >> 2) * lt::K_STAGES * KV_HALF + (ks & 3) * 32) / 16, idesc, ks > 0);
+          for (int t = 0; t < run; ++t) {
+            umma_commit(bar(lt::B_K_EMPTY + rk.stage));
+            rk.next(lt::K_STAGES);
+          }
+          j += run;
         }
         umma_commit(bar(lt::B_S_FULL + buf));
         ++cc;
@@ -817,9 +843,9 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
           seg += ceil16(len);
         }
       }
-      const int wlo = __reduce_min_sync(0xffffffffu, olo);
-      const int whi = __reduce_max_sync(0xffffffffu, ohi);
-      auto chunk_live = [&](int c0) { return c0 < m || (c0 <= whi && c0 + 31 >= wlo); };
+      // every 32-column chunk of S is read and put through the mask: a chunk no
+      // row of the warp sees contributes -inf to the maximum and exact zeros to P
+      // and to the sum, so skipping it would not change a bit
       auto vis_mask = [&](int c0) { return bits_in(-c0, m - c0) | bits_in(olo - c0, ohi + 1 - c0); };
       // ---- pass A: the row maximum, chunk by chunk
       float mx = -INFINITY;
@@ -830,12 +856,14 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
           break;
         }
         tc_fence_after();
-        for (int c0 = c * lt::CH; c0 < min(ncol, c * lt::CH + lt::CH); c0 += 32) {
-          if (!chunk_live(c0)) continue;
-          uint32_t v[32];
-          tmem_ld32(lane_base + lt::S_COL + lt::CH * buf + (c0 - c * lt::CH), v);
+        for (int c0 = c * lt::CH; c0 < min(ncol, c * lt::CH + lt::CH); c0 += KBLK) {
+          const uint32_t sb = lane_base + lt::S_COL + lt::CH * buf + (c0 - c * lt::CH);
+          uint32_t v0[32], v1[32];
+          tmem_ld32(sb, v0);
+          tmem_ld32(sb + 32, v1);
           tmem_ld_wait();
-          mx = fmaxf(mx, masked_max32(v, vis_mask(c0)));
+          mx = fmaxf(mx, masked_max32(v0, vis_mask(c0)));
+          mx = fmaxf(mx, masked_max32(v1, vis_mask(c0 + 32)));
         }
         tc_fence_before();
         __syncwarp();
@@ -858,21 +886,16 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
             ok = false;
             break;
           }
-#pragma unroll
-          for (int hf = 0; hf < 2; ++hf) {
-            const int cb = j * KBLK + 32 * hf;
-            uint32_t pk[16];
-            if (chunk_live(cb)) {
-              uint32_t v[32];
-              tmem_ld32(lane_base + lt::S_COL + lt::CH * buf + (cb - c * lt::CH), v);
-              tmem_ld_wait();
-              sum = exp_pack(v, vis_mask(cb), scale_log2, mxs, sum, pk);
-            } else {
-#pragma unroll
-              for (int q = 0; q < 16; ++q) pk[q] = 0u;
-            }
-            tmem_st16(lane_base + lt::P_COL + 32 * rp.stage + 16 * hf, pk);
-          }
+          const int cb = j * KBLK;
+          const uint32_t sb = lane_base + lt::S_COL + lt::CH * buf + (cb - c * lt::CH);
+          uint32_t v0[32], v1[32], pk[16];
+          tmem_ld32(sb, v0);
+          tmem_ld32(sb + 32, v1);
+          tmem_ld_wait();
+          sum = exp_pack(v0, vis_mask(cb), scale_log2, mxs, sum, pk);
+          tmem_st16(lane_base + lt::P_COL + 32 * rp.stage, pk);
+          sum = exp_pack(v1, vis_mask(cb + 32), scale_log2, mxs, sum, pk);
+          tmem_st16(lane_base + lt::P_COL + 32 * rp.stage + 16, pk);
           tmem_st_wait();
           tc_fence_before();
           __syncwarp();
@@ -892,16 +915,18 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
       const float inv = sum > 0.f ? 1.f / sum : 0.f;
 #pragma unroll 1
       for (int h = 0; h < 2; ++h) {
+        uint32_t v2[2][32];
+        tmem_ld32(lane_base + lt::O_COL + 64 * h, v2[0]);
+        tmem_ld32(lane_base + lt::O_COL + 64 * h + 32, v2[1]);
+        tmem_ld_wait();
+        if (h == 1) {  // O is out of TMEM
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar(lt::B_O_FREE));
+        }
 #pragma unroll
         for (int c2 = 0; c2 < 2; ++c2) {
-          uint32_t v[32];
-          tmem_ld32(lane_base + lt::O_COL + 64 * h + 32 * c2, v);
-          tmem_ld_wait();
-          if (h == 1 && c2 == 1) {  // O is out of TMEM
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(lt::B_O_FREE));
-          }
+          const uint32_t* v = v2[c2];
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const uint32_t* x = v + 8 * q;
