@@ -36,6 +36,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "scored query-doc pairs/sec at 1 GB300 (Qwen3-8B shape, m=64); p50 batch latency"
+NOMINAL_HBM_GBS = 7900.0  # GB300 HBM3e data-sheet bandwidth, printed beside the measured-peak fractions
 
 
 # Short numbers for the measured workloads: 0 the 2-layer Qwen3-0.6B-width case, 1 Qwen3-0.6B,
@@ -402,7 +403,8 @@ def run_dopr(args, rank, world, local_rank, dist):
             tf = v["flops"] / t_s / 1e12
             gbs = v["bytes"] / t_s / 1e9
             t_roof = max(v["flops"] / (peaks["bf16_tflops_sustained"] * 1e12), v["bytes"] / (peaks["hbm_gbs"] * 1e9))
-            ent.update({"tflops": tf, "gbs": gbs, "roofline_frac": t_roof / t_s})
+            ent.update({"tflops": tf, "gbs": gbs, "roofline_frac": t_roof / t_s,
+                        "gbs_frac_of_nominal_hbm": gbs / NOMINAL_HBM_GBS})
         kernels[name] = ent
     gpu_launches = sum(v["launches"] for v in prof.values())
 
