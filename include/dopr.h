@@ -48,7 +48,11 @@ typedef enum {
     DOPR_ERR_CUDA = 5,          /* a CUDA runtime/driver call failed          */
     DOPR_ERR_TIMEOUT = 6,       /* a bounded device wait ran out; the result
                                    of that call is invalid, the context is not */
-    DOPR_ERR_UNSUPPORTED = 7    /* a shape this build does not handle         */
+    DOPR_ERR_UNSUPPORTED = 7,   /* a shape this build does not handle         */
+    DOPR_ERR_INTERNAL = 8       /* a checked build (DOPR_CHECKED) met an index
+                                   outside its buffer and skipped the access:
+                                   a library defect; the call's outputs are
+                                   invalid, the context is not               */
 } dopr_status;
 
 /*

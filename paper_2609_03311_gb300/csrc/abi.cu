@@ -275,6 +275,7 @@ dopr_status map_device_error(int e) {
   if (e & DEV_ERR_BAD_TOKEN) return fail(DOPR_ERR_INVALID_ARG, "a token id is outside [0, vocab)");
   if (e & DEV_ERR_BAD_OFFSETS) return fail(DOPR_ERR_INVALID_ARG, "q_offsets must start at 0 and not decrease");
   if (e & DEV_ERR_POSITION) return fail(DOPR_ERR_INVALID_ARG, "m + query length + 1 exceeds max_position");
+  if (e & DEV_ERR_BOUNDS) return fail(DOPR_ERR_INTERNAL, "checked build: an index outside its buffer (access skipped)");
   return DOPR_OK;
 }
 
@@ -535,6 +536,7 @@ dopr_status run_packer(Model* m, Store* s, int32_t n, const int32_t* dqo, const 
 // the last layer stops there.
 struct BuildArgs {
   const bf16* x;  // device, [total rows][hidden]
+  int64_t rows;   // its rows
 };
 
 // Key token selection mode of run_layers: the packed tokens are documents'
@@ -545,6 +547,7 @@ struct BuildArgs {
 struct SelectState {
   int top_k, top_p;
   float* A;        // device, the largest chunk's sum of n^2
+  int64_t a_elems;  // floats in A
   int64_t* a_off;  // device, per chunk document
   float* u;        // device, [all tokens]
   int32_t* positions;
@@ -583,11 +586,19 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     const auto op = gemm_cost(T, H, m->o_dim, T * H * 10.0);
     const auto gu = gemm_cost(T, 2.0 * F, H, T * F * 2.0);
     const auto dn = gemm_cost(T, H, F, T * H * 10.0);
+    Extents ext;  // what the index tests of a checked build compare against
+    ext.err = w.err;
+    ext.rows = Tc;
+    ext.table_rows = build ? build->rows : c.vocab;
+    ext.pool_rows = s->pool_rows;
+    ext.rope_rows = c.max_position;
+    ext.a_elems = sel ? sel->a_elems : 0;
     CUDA_TRY(prof_launch(m, K_EMBED_NORM, 1, 0.0, T * H * 8.0, st, [&] {
       return launch_embed(w.tok_id + t0, Tc, build ? build->x : m->embed, m->attn_norm, H, c.rms_eps, w.r, w.xn,
-                          w.ss_e, st);
+                          w.ss_e, ext, st);
     }));
     GemmParams base{};
+    base.ext = ext;
     base.M = Tc;
     base.norm_dim = H;
     base.eps = c.rms_eps;
@@ -619,6 +630,7 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     ta.Hq = Hq;
     ta.Hkv = Hkv;
     ta.err = w.err;
+    ta.ext = ext;
     AttnTcArgs tl = ta;  // the long tiles, stored after every short tile
     tl.tiles = w.tiles + plan.n_tiles + plan.chunk_ltile[ci];
     tl.n_units = n_ltiles * Hkv;
@@ -656,7 +668,7 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       if (build) {  // this layer's keys and values are the document's stored prefix states
         CUDA_TRY(prof_launch(m, K_PREFIX_STORE, 1, 0.0, T * 2.0 * Hkv * HEAD_DIM * 2 * 2, st, [&] {
           return launch_prefix_store(w.qkv, m->qkv_dim, Tc, t0, Hq, Hkv, w.tok_pair, w.tok_pos, w.sorted_slot,
-                                     s->d_slot_row, s->d_slot_m, l, reinterpret_cast<f16*>(s->pool), st);
+                                     s->d_slot_row, s->d_slot_m, l, reinterpret_cast<f16*>(s->pool), ext, st);
         }));
         if (final_layer) continue;
       }
@@ -679,6 +691,7 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
         sa.u = sel->u + t0;
         sa.positions = sel->positions;
         sa.x = sel->x;
+        sa.ext = ext;
         std::vector<int64_t> aoff(s1 - s0);
         int64_t acc = 0;
         for (int32_t d = s0; d < s1; ++d) {
@@ -707,6 +720,7 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       aa.score_only = last ? 1 : 0;
       aa.pair_base = s0;
       aa.err = w.err;
+      aa.ext = ext;
       const int attn_launches = (!last && ta.n_units > 0 ? 1 : 0) + (!last && tl.n_units > 0 ? 1 : 0) +
                                 (aa.n_items > 0 ? 1 : 0);
       CUDA_TRY(prof_launch(m, K_ATTENTION, attn_launches, last ? attn_flops_last : attn_flops,
@@ -732,7 +746,8 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       int rows = Tc;
       if (last) {
         CUDA_TRY(prof_launch(m, K_SCORE, 1, 0.0, np * (H * 8.0 + ss_pre_parts * 8.0), st, [&] {
-          return launch_gather_score_rows(w.r, ss_pre, H, ss_pre_parts, w.tok_off, t0, s0, s1, w.r_s, w.ss_s, st);
+          return launch_gather_score_rows(w.r, ss_pre, H, ss_pre_parts, w.tok_off, t0, s0, s1, w.r_s, w.ss_s, ext,
+                                          st);
         }));
         ss_pre = w.ss_s;
         resid = w.r_s;
@@ -788,12 +803,12 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
                              [&] {
                                return launch_score_mlp(w.r_s, H, w.tok_off, t0, s0, s1, 1, w.perm, m->final_norm,
                                                        c.rms_eps, m->mlp_width, m->mlp_act, m->mlp_w1, m->mlp_b1,
-                                                       m->mlp_w2, m->mlp_b2, d_scores, st);
+                                                       m->mlp_w2, m->mlp_b2, d_scores, ext, st);
                              }));
       } else {
         CUDA_TRY(prof_launch(m, K_SCORE, 1, 4.0 * H * (s1 - s0), (s1 - s0) * (H * 4.0 + 4.0), st, [&] {
           return launch_score(w.r_s, H, w.tok_off, t0, s0, s1, 1, w.perm, m->final_norm, m->score_head, c.rms_eps,
-                              d_scores, st);
+                              d_scores, ext, st);
         }));
       }
     } else if (sel) {  // final states of the selected rows: the representations C_d
@@ -805,6 +820,7 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       sa.top_k = sel->top_k;
       sa.positions = sel->positions;
       sa.x = sel->x;
+      sa.ext = ext;
       CUDA_TRY(launch_select_gather(sa, w.r, H, m->final_norm, c.rms_eps, st));
     }
   }
@@ -1252,7 +1268,7 @@ dopr_status dopr_build_prefixes(dopr_model* m, dopr_store* s, int32_t n_docs, co
       dx = stage;
     }
     CUDA_TRY(cudaMemsetAsync(w.err, 0, sizeof(int), st));
-    BuildArgs b{dx};
+    BuildArgs b{dx, (int64_t)rows};
     const dopr_status rs = run_layers(m, s, plan, nullptr, st, &b);
     cudaError_t e = cudaMemcpyAsync(w.h_err, w.err, sizeof(int), cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
@@ -1342,7 +1358,7 @@ dopr_status dopr_select_prefix_inputs(dopr_model* m, int32_t n_docs, const int32
   }
   STATUS_TRY(ap.upload(w, plan, 0, st));
   // selection buffers for this call
-  SelectState sel{top_k, top_p, nullptr, nullptr, nullptr, nullptr, nullptr};
+  SelectState sel{top_k, top_p, nullptr, a_max, nullptr, nullptr, nullptr, nullptr};
   auto cleanup = [&] {
     dev_free(sel.A); dev_free(sel.a_off); dev_free(sel.u); dev_free(sel.positions); dev_free(sel.x);
   };

@@ -21,7 +21,24 @@ enum : int {
   DEV_ERR_BAD_TOKEN = 1 << 3,    // token id outside [0, vocab)
   DEV_ERR_BAD_OFFSETS = 1 << 4,  // q_offsets decreasing / not starting at 0
   DEV_ERR_POSITION = 1 << 5,     // m + query length reaches max_position
+  DEV_ERR_BOUNDS = 1 << 6,       // checked build: an index outside its buffer (the access was skipped)
 };
+
+// Index tests of checked builds (compiled with -DDOPR_CHECKED).  index_ok(err,
+// i, n) is true when 0 <= i < n; otherwise it sets DEV_ERR_BOUNDS in *err and
+// returns false, and the caller skips (or, for a TMA copy, which the hardware
+// bounds itself, only reports) the access.  Plain builds take every index as in
+// range and compile the tests away.
+#ifdef DOPR_CHECKED
+constexpr bool kCheckedBuild = true;
+#else
+constexpr bool kCheckedBuild = false;
+#endif
+__device__ __forceinline__ bool index_ok(int* err, int64_t i, int64_t n) {
+  if (!kCheckedBuild || (i >= 0 && i < n)) return true;
+  if (err) atomicOr(err, DEV_ERR_BOUNDS);
+  return false;
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));

@@ -22,6 +22,17 @@ constexpr int MAX_PREFIX = 256;       // largest m the store accepts
 constexpr int ATTN_MAX_PAIRS = 8;     // pairs of one doc per attention work item
 constexpr uint64_t WAIT_TIMEOUT_NS = 4000000000ull;  // bounded device waits: 4 s
 
+// Buffer extents the index tests of a checked build compare against (see
+// index_ok in device_common.cuh); plain builds carry them unused.
+struct Extents {
+  int* err = nullptr;      // the call's device error word
+  int64_t rows = 0;        // rows of the chunk's activation buffers (packed tokens)
+  int64_t table_rows = 0;  // rows of the table a gather reads (embedding, or a build's input vectors)
+  int64_t pool_rows = 0;   // 256-byte rows of the store pool
+  int64_t rope_rows = 0;   // positions of the RoPE table
+  int64_t a_elems = 0;     // floats of the key token selection's attention matrices
+};
+
 // One attention work item: consecutive sorted pairs that share a document.
 struct AttnItem {
   int32_t pair_begin, pair_end;  // sorted pair indices [begin, end)
@@ -197,6 +208,7 @@ struct GemmParams {
   int q_cols, k_cols;
   int* err;
   uint64_t timeout_ns;
+  Extents ext;
 };
 cudaError_t gemm_setup();
 // C[M][N] = A[M][K] * B[N][K]^T followed by the epilogue `epi`.
@@ -207,21 +219,23 @@ cudaError_t launch_gemm(int epi, const CUtensorMap& tmA, const CUtensorMap& tmB,
 // r[t] = E[tok_id[t]] (fp32), ss[t] = sum(r[t]^2), xn[t] = f16(r[t] * rsqrt(ss[t]/H + eps) * gain):
 // the embedding and the first RMSNorm.
 cudaError_t launch_embed(const int32_t* tok_id, int T, const bf16* embed, const bf16* gain, int H, float eps, float* r,
-                         f16* xn, float* ss, cudaStream_t st);
+                         f16* xn, float* ss, const Extents& ext, cudaStream_t st);
 // In place: n bf16 values -> fp16 (saturating at +-65504).
 cudaError_t launch_bf16_to_f16(void* buf, int64_t n, cudaStream_t st);
 // Score head over sorted pairs [p_begin, p_end): the score-token row of pair s is
 // r[tok_off[s+1]-1-tok0], or r[s - p_begin] when `compact` is set.
 cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end, int compact,
                          const int32_t* perm, const bf16* gain, const bf16* head, float eps, float* scores,
-                         cudaStream_t st);
+                         const Extents& ext, cudaStream_t st);
 // Compact the score-token rows of sorted pairs [p_begin, p_end): dst_r[i] = r[row(i)] (H floats) and
 // dst_ss[i] = ss[row(i)] (parts floats), row(i) = tok_off[p_begin+i+1]-1-tok0.
 cudaError_t launch_score_mlp(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end,
                              int compact, const int32_t* perm, const bf16* gain, float eps, int width, int act,
-                             const bf16* w1, const bf16* b1, const bf16* w2, float b2, float* scores, cudaStream_t st);
+                             const bf16* w1, const bf16* b1, const bf16* w2, float b2, float* scores,
+                             const Extents& ext, cudaStream_t st);
 cudaError_t launch_gather_score_rows(const float* r, const float* ss, int H, int parts, const int32_t* tok_off,
-                                     int tok0, int p_begin, int p_end, float* dst_r, float* dst_ss, cudaStream_t st);
+                                     int tok0, int p_begin, int p_end, float* dst_r, float* dst_ss, const Extents& ext,
+                                     cudaStream_t st);
 // [m][Hkv][128] bf16 -> [Hkv][m][128] fp16 for K and V; *range |= 1 when a value
 // is not finite or exceeds the fp16 range (|x| > 65504).
 cudaError_t launch_store_transpose(const bf16* k, const bf16* v, int m, int Hkv, f16* dk, f16* dv, int* range,
@@ -243,6 +257,7 @@ struct AttnArgs {
   int score_only;  // 1: only each pair's score-token rows, written to out row (pair - pair_base)
   int pair_base;
   int* err;
+  Extents ext;
 };
 cudaError_t attn_setup();
 cudaError_t launch_attention(const CUtensorMap& tm_pool, const AttnArgs& a, cudaStream_t st);
@@ -255,6 +270,7 @@ struct AttnTcArgs {
   int ld_out;
   int layer, Hq, Hkv;
   int* err;
+  Extents ext;
 };
 // Q rows per head in a 128-row tile; 0 when the group size does not divide 128 into boxes of >= 8 rows.
 inline int attn_tc_rows_per_head(int G) { return (G >= 1 && G <= 16 && 128 % G == 0) ? 128 / G : 0; }
@@ -316,6 +332,7 @@ struct SelectArgs {
   float* u;                 // salience of chunk row t at u[t]
   int32_t* positions;       // [all documents][top_k]
   bf16* x;                  // [all documents][top_k][hidden]
+  Extents ext;
 };
 cudaError_t select_setup();
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
@@ -324,7 +341,7 @@ cudaError_t launch_select_gather(const SelectArgs& a, const float* r, int H, con
 // Prefix build: K/V rows of chunk tokens [0, T) (packed tokens t0 + t) into the store pool.
 cudaError_t launch_prefix_store(const f16* qkv, int ld_qkv, int T, int t0, int Hq, int Hkv, const int32_t* tok_pair,
                                 const int32_t* tok_pos, const int32_t* pair_slot, const int64_t* slot_row,
-                                const int32_t* slot_m, int layer, f16* pool, cudaStream_t st);
+                                const int32_t* slot_m, int layer, f16* pool, const Extents& ext, cudaStream_t st);
 cudaError_t launch_wait_timeout_probe(int* err, uint64_t timeout_ns, cudaStream_t st);
 
 }  // namespace dopr

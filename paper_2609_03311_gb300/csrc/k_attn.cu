@@ -148,10 +148,10 @@ __device__ __forceinline__ void load_q(const AttnArgs& a, const PairGeom& pg, in
   const int ra = row0 + (lane >> 2), rb = ra + 8;
   const uint32_t* qa = nullptr;
   const uint32_t* qb = nullptr;
-  if (ra < pg.R)
+  if (ra < pg.R && index_ok(a.ext.err, pg.tb + ra / G, a.ext.rows))
     qa = reinterpret_cast<const uint32_t*>(a.qkv + static_cast<int64_t>(pg.tb + ra / G) * a.ld_qkv +
                                            (g * G + ra % G) * HEAD_DIM);
-  if (rb < pg.R)
+  if (rb < pg.R && index_ok(a.ext.err, pg.tb + rb / G, a.ext.rows))
     qb = reinterpret_cast<const uint32_t*>(a.qkv + static_cast<int64_t>(pg.tb + rb / G) * a.ld_qkv +
                                            (g * G + rb % G) * HEAD_DIM);
   const int t = lane & 3;
@@ -184,9 +184,9 @@ __device__ __forceinline__ void store_tile(const AttnArgs& a, const PairGeom& pg
 #pragma unroll
   for (int hr = 0; hr < 2; ++hr) {
     const int row = row0 + (lane >> 2) + hr * 8;
-    if (row < pg.R) {
-      const int j = row / G, hh = row % G;
-      const int orow = a.score_only ? s - a.pair_base : pg.tb + j;
+    const int orow = a.score_only ? s - a.pair_base : pg.tb + row / G;
+    if (row < pg.R && index_ok(a.ext.err, orow, a.ext.rows)) {
+      const int hh = row % G;
       f16* dst = a.out + static_cast<int64_t>(orow) * a.ld_out + (g * G + hh) * HEAD_DIM + (lane & 3) * 2;
       const float inv = hr ? inv1 : inv0;
 #pragma unroll
@@ -205,7 +205,7 @@ __device__ __forceinline__ void load_own(const AttnArgs& a, int g, uint32_t sOK,
   const int rows = min(OWN_ROWS, count + 16);
   for (int idx = tid; idx < rows * 32; idx += THREADS) {
     const int kv = idx & 1, rc = idx >> 1, r = rc >> 4, c = rc & 15;
-    const bool ok = r < count;
+    const bool ok = r < count && index_ok(a.ext.err, row_begin + r, a.ext.rows);
     const f16* src = a.qkv + static_cast<int64_t>(row_begin + (ok ? r : 0)) * a.ld_qkv + (kv ? vcol : kcol) + c * 8;
     cp_async16((kv ? sOV : sOK) + off_own(r, c), src, ok);
   }
@@ -241,6 +241,10 @@ __global__ void __launch_bounds__(THREADS, DOPR_ATTN_MIN_BLOCKS) k_attn(const __
       const int64_t base = a.slot_row[item.slot];
       const int rowK = static_cast<int>(base + (static_cast<int64_t>(a.layer) * 2 * a.Hkv + g) * m);
       const int rowV = static_cast<int>(base + ((static_cast<int64_t>(a.layer) * 2 + 1) * a.Hkv + g) * m);
+      if (kCheckedBuild) {  // report only: the tensor map bounds the copies itself
+        index_ok(a.ext.err, rowK + m - 1, a.ext.pool_rows);
+        index_ok(a.ext.err, rowV + m - 1, a.ext.pool_rows);
+      }
       mbar_arrive_expect_tx(bar, static_cast<uint32_t>(nbox) * 4u * BOX_BYTES);
       for (int b = 0; b < nbox; ++b)
         for (int h = 0; h < 2; ++h) {

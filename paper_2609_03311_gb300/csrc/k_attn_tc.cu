@@ -254,6 +254,11 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int nb = (n_keys + KBLK - 1) / KBLK;
         const int pool_row = static_cast<int>(tp->pool_base + ((static_cast<int64_t>(a.layer) * 2 + kv) * a.Hkv + g) * m);
         const int col0 = (a.Hq + kv * a.Hkv + g) * HEAD_DIM;
+        if (kCheckedBuild) {  // report only: the tensor maps bound every copy themselves
+          index_ok(a.ext.err, tok_begin + seg_start(tp->seg[0]), a.ext.rows);
+          index_ok(a.ext.err, tok_begin + tp->n_tok - 1, a.ext.rows);
+          if (m > 0) index_ok(a.ext.err, pool_row + m - 1, a.ext.pool_rows);
+        }
         int si = 0, k = 0, key = pre64;  // own-key cursor: segment, row within it, key column
         int sv = tp->seg[0];
         for (int j = 0; j < nb; ++j) {
@@ -535,7 +540,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const int rr = it * 4 + (lane >> 3), ch = lane & 7;
           const int row = quarter * 32 + rr;  // tile row
           const int j2 = row % TT;
-          if (j2 < n_tok) {
+          if (j2 < n_tok && index_ok(a.ext.err, tp->tok_begin + j2, a.ext.rows)) {
             const uint4 x = *reinterpret_cast<const uint4*>(stg + rr * 128 + ((ch ^ (rr & 7)) << 4));
             *reinterpret_cast<uint4*>(a.out + static_cast<int64_t>(tp->tok_begin + j2) * a.ld_out +
                                       (g * G + row / TT) * HEAD_DIM + 64 * h + ch * 8) = x;
@@ -667,6 +672,11 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
         st.sv = tp->seg[0];
         st.pool_row = static_cast<int>(tp->pool_base + ((static_cast<int64_t>(a.layer) * 2 + kv) * a.Hkv + g) * tp->m);
         st.col0 = (a.Hq + kv * a.Hkv + g) * HEAD_DIM;
+        if (kCheckedBuild) {  // report only: the tensor maps bound every copy themselves
+          index_ok(a.ext.err, tp->tok_begin + seg_start(tp->seg[0]), a.ext.rows);
+          index_ok(a.ext.err, tp->tok_begin + tp->n_tok - 1, a.ext.rows);
+          if (tp->m > 0) index_ok(a.ext.err, st.pool_row + tp->m - 1, a.ext.pool_rows);
+        }
         return st;
       };
       auto issue_block = [&](const AttnTile* tp, Stream& st, int j) -> bool {
@@ -945,7 +955,7 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
           const int rr = it * 4 + (lane >> 3), ch = lane & 7;
           const int row = quarter * 32 + rr;  // tile row
           const int j2 = row % TT;
-          if (j2 < n_tok) {
+          if (j2 < n_tok && index_ok(a.ext.err, tp->tok_begin + j2, a.ext.rows)) {
             const uint4 x = *reinterpret_cast<const uint4*>(stg + rr * 128 + ((ch ^ (rr & 7)) << 4));
             *reinterpret_cast<uint4*>(a.out + static_cast<int64_t>(tp->tok_begin + j2) * a.ld_out +
                                       (g * G + row / TT) * HEAD_DIM + 64 * h + ch * 8) = x;

@@ -17,10 +17,12 @@ constexpr int ROW_WARPS = 8;  // warps per block for row kernels
 // xn = f16(r * rsqrt(ss/H + eps) * g).  The row is read twice (the second read hits L1).
 __global__ void __launch_bounds__(ROW_WARPS * 32)
     k_embed(const int32_t* __restrict__ tok_id, int T, const bf16* __restrict__ embed, const bf16* __restrict__ gain,
-            int H, float eps, float* __restrict__ r, f16* __restrict__ xn, float* __restrict__ ss_out) {
+            int H, float eps, float* __restrict__ r, f16* __restrict__ xn, float* __restrict__ ss_out, Extents ext) {
   const int row = blockIdx.x * ROW_WARPS + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (row >= T) return;
-  const bf16* e = embed + static_cast<int64_t>(tok_id[row]) * H;
+  const int64_t id = tok_id[row];
+  if (!index_ok(ext.err, id, ext.table_rows) || !index_ok(ext.err, row, ext.rows)) return;
+  const bf16* e = embed + id * H;
   float* rr = r + static_cast<int64_t>(row) * H;
   f16* xr = xn + static_cast<int64_t>(row) * H;
   float ss = 0.f;
@@ -69,10 +71,11 @@ __global__ void k_bf16_to_f16(uint32_t* __restrict__ buf, int64_t n_words) {
 __global__ void __launch_bounds__(ROW_WARPS * 32)
     k_score(const float* __restrict__ r, int H, const int32_t* __restrict__ tok_off, int tok0, int p_begin, int p_end,
             int compact, const int32_t* __restrict__ perm, const bf16* __restrict__ gain,
-            const bf16* __restrict__ head, float eps, float* __restrict__ scores) {
+            const bf16* __restrict__ head, float eps, float* __restrict__ scores, Extents ext) {
   const int s = p_begin + blockIdx.x * ROW_WARPS + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (s >= p_end) return;
   const int64_t row = compact ? s - p_begin : tok_off[s + 1] - 1 - tok0;
+  if (!index_ok(ext.err, row, ext.rows)) return;
   const float* x = r + row * H;
   float ss = 0.f;
   for (int c = lane * 4; c < H; c += 128) {
@@ -111,11 +114,12 @@ __global__ void __launch_bounds__(MLP_THREADS)
     k_score_mlp(const float* __restrict__ r, int H, const int32_t* __restrict__ tok_off, int tok0, int p_begin,
                 int compact, const int32_t* __restrict__ perm, const bf16* __restrict__ gain, float eps, int width,
                 int act, const bf16* __restrict__ w1, const bf16* __restrict__ b1, const bf16* __restrict__ w2,
-                float b2, float* __restrict__ scores) {
+                float b2, float* __restrict__ scores, Extents ext) {
   extern __shared__ float hn[];  // [H], then 32 partial sums
   float* red = hn + H;
   const int s = p_begin + blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t row = compact ? s - p_begin : tok_off[s + 1] - 1 - tok0;
+  if (!index_ok(ext.err, row, ext.rows)) return;  // uniform across the block
   const float* x = r + row * H;
   float ss = 0.f;
   for (int c = threadIdx.x; c < H; c += blockDim.x) ss += x[c] * x[c];
@@ -152,10 +156,11 @@ __global__ void __launch_bounds__(MLP_THREADS)
 __global__ void __launch_bounds__(ROW_WARPS * 32)
     k_gather_score_rows(const float* __restrict__ r, const float* __restrict__ ss, int H, int parts,
                         const int32_t* __restrict__ tok_off, int tok0, int p_begin, int p_end,
-                        float* __restrict__ dst_r, float* __restrict__ dst_ss) {
+                        float* __restrict__ dst_r, float* __restrict__ dst_ss, Extents ext) {
   const int i = blockIdx.x * ROW_WARPS + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (p_begin + i >= p_end) return;
   const int64_t row = tok_off[p_begin + i + 1] - 1 - tok0;
+  if (!index_ok(ext.err, row, ext.rows) || !index_ok(ext.err, i, ext.rows)) return;
   const float4* src = reinterpret_cast<const float4*>(r + row * H);
   float4* dst = reinterpret_cast<float4*>(dst_r + static_cast<int64_t>(i) * H);
   for (int c = lane; c < H / 4; c += 32) dst[c] = src[c];
@@ -199,7 +204,7 @@ __global__ void k_store_transpose(const uint4* __restrict__ k, const uint4* __re
 __global__ void k_prefix_store(const f16* __restrict__ qkv, int ld_qkv, int T, int t0, int Hq, int Hkv,
                                const int32_t* __restrict__ tok_pair, const int32_t* __restrict__ tok_pos,
                                const int32_t* __restrict__ pair_slot, const int64_t* __restrict__ slot_row,
-                               const int32_t* __restrict__ slot_m, int layer, f16* __restrict__ pool) {
+                               const int32_t* __restrict__ slot_m, int layer, f16* __restrict__ pool, Extents ext) {
   const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (w >= static_cast<int64_t>(T) * Hkv * 2) return;
@@ -209,6 +214,7 @@ __global__ void k_prefix_store(const f16* __restrict__ qkv, int ld_qkv, int T, i
   const int p = tok_pair[t0 + t], j = tok_pos[t0 + t];
   const int slot = pair_slot[p];
   const int64_t row = slot_row[slot] + (static_cast<int64_t>(layer * 2 + kv) * Hkv + g) * slot_m[slot] + j;
+  if (!index_ok(ext.err, j, slot_m[slot]) || !index_ok(ext.err, row, ext.pool_rows)) return;
   const uint2* src = reinterpret_cast<const uint2*>(qkv + static_cast<int64_t>(t) * ld_qkv + (Hq + kv * Hkv + g) * HEAD_DIM);
   reinterpret_cast<uint2*>(pool + row * HEAD_DIM)[lane] = src[lane];
 }
@@ -231,9 +237,9 @@ inline int blocks_for(int64_t rows) { return static_cast<int>((rows + ROW_WARPS 
 }  // namespace
 
 cudaError_t launch_embed(const int32_t* tok_id, int T, const bf16* embed, const bf16* gain, int H, float eps, float* r,
-                         f16* xn, float* ss, cudaStream_t st) {
+                         f16* xn, float* ss, const Extents& ext, cudaStream_t st) {
   if (T <= 0) return cudaSuccess;
-  k_embed<<<blocks_for(T), ROW_WARPS * 32, 0, st>>>(tok_id, T, embed, gain, H, eps, r, xn, ss);
+  k_embed<<<blocks_for(T), ROW_WARPS * 32, 0, st>>>(tok_id, T, embed, gain, H, eps, r, xn, ss, ext);
   return cudaGetLastError();
 }
 
@@ -247,27 +253,29 @@ cudaError_t launch_bf16_to_f16(void* buf, int64_t n, cudaStream_t st) {
 
 cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end, int compact,
                          const int32_t* perm, const bf16* gain, const bf16* head, float eps, float* scores,
-                         cudaStream_t st) {
+                         const Extents& ext, cudaStream_t st) {
   if (p_end <= p_begin) return cudaSuccess;
   k_score<<<blocks_for(p_end - p_begin), ROW_WARPS * 32, 0, st>>>(r, H, tok_off, tok0, p_begin, p_end, compact, perm,
-                                                                  gain, head, eps, scores);
+                                                                  gain, head, eps, scores, ext);
   return cudaGetLastError();
 }
 
 cudaError_t launch_score_mlp(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end,
                              int compact, const int32_t* perm, const bf16* gain, float eps, int width, int act,
-                             const bf16* w1, const bf16* b1, const bf16* w2, float b2, float* scores, cudaStream_t st) {
+                             const bf16* w1, const bf16* b1, const bf16* w2, float b2, float* scores,
+                             const Extents& ext, cudaStream_t st) {
   if (p_end <= p_begin) return cudaSuccess;
   k_score_mlp<<<p_end - p_begin, MLP_THREADS, (H + 32) * sizeof(float), st>>>(
-      r, H, tok_off, tok0, p_begin, compact, perm, gain, eps, width, act, w1, b1, w2, b2, scores);
+      r, H, tok_off, tok0, p_begin, compact, perm, gain, eps, width, act, w1, b1, w2, b2, scores, ext);
   return cudaGetLastError();
 }
 
 cudaError_t launch_gather_score_rows(const float* r, const float* ss, int H, int parts, const int32_t* tok_off,
-                                     int tok0, int p_begin, int p_end, float* dst_r, float* dst_ss, cudaStream_t st) {
+                                     int tok0, int p_begin, int p_end, float* dst_r, float* dst_ss,
+                                     const Extents& ext, cudaStream_t st) {
   if (p_end <= p_begin) return cudaSuccess;
   k_gather_score_rows<<<blocks_for(p_end - p_begin), ROW_WARPS * 32, 0, st>>>(r, ss, H, parts, tok_off, tok0, p_begin,
-                                                                              p_end, dst_r, dst_ss);
+                                                                              p_end, dst_r, dst_ss, ext);
   return cudaGetLastError();
 }
 
@@ -283,11 +291,11 @@ cudaError_t launch_store_transpose(const bf16* k, const bf16* v, int m, int Hkv,
 
 cudaError_t launch_prefix_store(const f16* qkv, int ld_qkv, int T, int t0, int Hq, int Hkv, const int32_t* tok_pair,
                                 const int32_t* tok_pos, const int32_t* pair_slot, const int64_t* slot_row,
-                                const int32_t* slot_m, int layer, f16* pool, cudaStream_t st) {
+                                const int32_t* slot_m, int layer, f16* pool, const Extents& ext, cudaStream_t st) {
   const int64_t threads = static_cast<int64_t>(T) * Hkv * 2 * 32;
   if (threads <= 0) return cudaSuccess;
   k_prefix_store<<<static_cast<unsigned>((threads + 255) / 256), 256, 0, st>>>(
-      qkv, ld_qkv, T, t0, Hq, Hkv, tok_pair, tok_pos, pair_slot, slot_row, slot_m, layer, pool);
+      qkv, ld_qkv, T, t0, Hq, Hkv, tok_pair, tok_pos, pair_slot, slot_row, slot_m, layer, pool, ext);
   return cudaGetLastError();
 }
 

@@ -46,7 +46,8 @@ __device__ __forceinline__ float block_reduce(float v, float* red, bool is_max) 
 __global__ void __launch_bounds__(PROB_THREADS) k_sal_probs(const f16* __restrict__ qkv, int ld_qkv, int Hq, int Hkv,
                                                             const int32_t* __restrict__ tok_pair,
                                                             const int32_t* __restrict__ tok_off, int t0, int p0,
-                                                            const int64_t* __restrict__ a_off, float* __restrict__ A) {
+                                                            const int64_t* __restrict__ a_off, float* __restrict__ A,
+                                                            Extents ext) {
   extern __shared__ float sm[];
   float* q = sm;                  // [128]
   float* red = q + HEAD_DIM;      // [32]
@@ -57,6 +58,10 @@ __global__ void __launch_bounds__(PROB_THREADS) k_sal_probs(const f16* __restric
   const int ts = tok_off[p] - t0, n = tok_off[p + 1] - tok_off[p];
   const int jt = t - ts;          // row within the document
   const int G = Hq / Hkv;
+  // block-uniform: the document's rows in the chunk and its row of A-bar
+  if (!index_ok(ext.err, ts, ext.rows) || !index_ok(ext.err, ts + n - 1, ext.rows) ||
+      !index_ok(ext.err, a_off[p - p0] + static_cast<int64_t>(jt + 1) * n - 1, ext.a_elems))
+    return;
   const float scale = rsqrtf(static_cast<float>(HEAD_DIM));
   for (int i = threadIdx.x; i <= jt; i += blockDim.x) acc[i] = 0.f;
   for (int h = 0; h < Hq; ++h) {
@@ -129,7 +134,7 @@ __global__ void __launch_bounds__(SORT_THREADS) k_sal_colstat(const int32_t* __r
                                                               const int32_t* __restrict__ tok_off, int t0, int p0,
                                                               const int64_t* __restrict__ a_off,
                                                               const float* __restrict__ A, int top_p,
-                                                              float* __restrict__ u) {
+                                                              float* __restrict__ u, Extents ext) {
   __shared__ float v[SEL_MAX_N];
   __shared__ float red[32];
   const int t = blockIdx.x;
@@ -137,6 +142,7 @@ __global__ void __launch_bounds__(SORT_THREADS) k_sal_colstat(const int32_t* __r
   const int ts = tok_off[p] - t0, n = tok_off[p + 1] - tok_off[p];
   const int i = t - ts;
   const int cnt = n - i, k = min(top_p, cnt);
+  if (!index_ok(ext.err, a_off[p - p0] + static_cast<int64_t>(n) * n - 1, ext.a_elems)) return;  // block-uniform
   const float* col = A + a_off[p - p0] + i;
   float sum = 0.f;
   if (k == cnt) {
@@ -182,7 +188,7 @@ __global__ void __launch_bounds__(SORT_THREADS) k_sal_topk(const int32_t* __rest
 // One warp per (document, selected slot): x = bf16(RMSNorm(r_row) * g_final), zeros for -1.
 __global__ void k_sal_gather(const float* __restrict__ r, int H, const int32_t* __restrict__ tok_off, int t0,
                              int p0, int n_docs, const int32_t* __restrict__ positions, int K,
-                             const bf16* __restrict__ gain, float eps, bf16* __restrict__ x) {
+                             const bf16* __restrict__ gain, float eps, bf16* __restrict__ x, Extents ext) {
   const int w = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (w >= n_docs * K) return;
   const int p = p0 + w / K, j = w % K;
@@ -192,7 +198,9 @@ __global__ void k_sal_gather(const float* __restrict__ r, int H, const int32_t* 
     for (int c = lane; c < H; c += 32) dst[c] = __float2bfloat16(0.f);
     return;
   }
-  const float* row = r + static_cast<int64_t>(tok_off[p] - t0 + pos) * H;
+  const int64_t rr = static_cast<int64_t>(tok_off[p] - t0) + pos;
+  if (!index_ok(ext.err, rr, ext.rows)) return;
+  const float* row = r + rr * H;
   float ss = 0.f;
   for (int c = lane; c < H; c += 32) ss += row[c] * row[c];
   ss = warp_sum(ss);
@@ -211,10 +219,11 @@ cudaError_t launch_select(const SelectArgs& a, cudaStream_t st) {
   if (a.n_rows <= 0) return cudaSuccess;
   const size_t smem = (HEAD_DIM + 32 + 2 * SEL_MAX_N) * sizeof(float);
   k_sal_probs<<<a.n_rows, PROB_THREADS, smem, st>>>(a.qkv, a.ld_qkv, a.Hq, a.Hkv, a.tok_pair, a.tok_off, a.t0, a.p0,
-                                                    a.a_off, a.A);
+                                                    a.a_off, a.A, a.ext);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_sal_colstat<<<a.n_rows, SORT_THREADS, 0, st>>>(a.tok_pair, a.tok_off, a.t0, a.p0, a.a_off, a.A, a.top_p, a.u);
+  k_sal_colstat<<<a.n_rows, SORT_THREADS, 0, st>>>(a.tok_pair, a.tok_off, a.t0, a.p0, a.a_off, a.A, a.top_p, a.u,
+                                                   a.ext);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   k_sal_topk<<<a.n_docs, SORT_THREADS, 0, st>>>(a.tok_off, a.t0, a.p0, a.u, a.top_k, a.positions);
   return cudaGetLastError();
@@ -225,7 +234,8 @@ cudaError_t launch_select_gather(const SelectArgs& a, const float* r, int H, con
   const int64_t threads = static_cast<int64_t>(a.n_docs) * a.top_k * 32;
   if (threads <= 0) return cudaSuccess;
   k_sal_gather<<<static_cast<unsigned>((threads + 255) / 256), 256, 0, st>>>(r, H, a.tok_off, a.t0, a.p0, a.n_docs,
-                                                                             a.positions, a.top_k, gain, eps, a.x);
+                                                                             a.positions, a.top_k, gain, eps, a.x,
+                                                                             a.ext);
   return cudaGetLastError();
 }
 

@@ -17,8 +17,10 @@ from . import build as _build
 
 _LIB = None
 
-OK, ERR_INVALID_ARG, ERR_UNKNOWN_DOC, ERR_INCOMPLETE, ERR_OUT_OF_MEMORY, ERR_CUDA, ERR_TIMEOUT, ERR_UNSUPPORTED = range(8)
-STATUS_NAMES = ["OK", "INVALID_ARG", "UNKNOWN_DOC", "INCOMPLETE", "OUT_OF_MEMORY", "CUDA", "TIMEOUT", "UNSUPPORTED"]
+(OK, ERR_INVALID_ARG, ERR_UNKNOWN_DOC, ERR_INCOMPLETE, ERR_OUT_OF_MEMORY, ERR_CUDA, ERR_TIMEOUT, ERR_UNSUPPORTED,
+ ERR_INTERNAL) = range(9)
+STATUS_NAMES = ["OK", "INVALID_ARG", "UNKNOWN_DOC", "INCOMPLETE", "OUT_OF_MEMORY", "CUDA", "TIMEOUT", "UNSUPPORTED",
+                "INTERNAL"]
 
 (W_EMBED, W_ATTN_NORM, W_Q, W_K, W_V, W_Q_NORM, W_K_NORM, W_O, W_MLP_NORM, W_GATE, W_UP, W_DOWN, W_FINAL_NORM,
  W_SCORE_HEAD) = range(14)
@@ -45,7 +47,8 @@ class ModelConfig(ctypes.Structure):
 
 
 def lib_path() -> str:
-    return _build.LIB
+    """The library this process loads: the checked build when DOPR_CHECKED=1."""
+    return _build.LIB_CHECKED if os.environ.get("DOPR_CHECKED") == "1" else _build.LIB
 
 
 def load():
