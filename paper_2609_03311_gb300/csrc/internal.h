@@ -43,8 +43,11 @@ struct AttnItem {
 // Tensor-core attention (k_attn_tc.cu).  A tile is up to 128 / G consecutive
 // packed tokens of pairs of one document; its keys are the prefix (ceil64(m)
 // columns) then one segment per pair it touches, from the pair's first token to
-// the tile's last, each padded to a multiple of 16 columns.  Pairs whose own
-// segment can exceed the key budget take the mma.sync kernel (k_attn.cu).
+// the tile's last, each padded to a multiple of 16 columns.  A tile keeps within
+// ATTN_TC_MAX_KEYS columns (k_attn_tc) unless its first token alone needs more
+// (a long tile, k_attn_tc_long, no key limit).  The mma.sync kernel (k_attn.cu)
+// takes the last layer's score-token rows, and every row when 128 / G gives no
+// tile shape.
 constexpr int ATTN_TC_MAX_KEYS = 256;
 constexpr int ATTN_TC_MAX_SEGS = 16;  // own segments are >= 16 columns each
 struct __align__(16) AttnTile {

@@ -19,8 +19,9 @@
 // than OWN_CAP stream their own keys in OWN_CAP chunks per 64-row group.
 // Scores and P.V use warp-level fp16 mma with fp32 accumulation (the store
 // keeps the prefix as fp16); row maxima and sums use quad shuffles.  This
-// kernel takes the pairs whose keys exceed the tensor-core kernel's budget and
-// the score-token rows of the last layer.
+// kernel takes the score-token rows of the last layer (one row per pair and
+// q head), and every row when the GQA group size gives the tensor-core
+// kernels no tile shape.
 #include <math.h>
 
 #include "device_common.cuh"
