@@ -591,14 +591,12 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     ext.rows = Tc;
     ext.table_rows = build ? build->rows : c.vocab;
     ext.pool_rows = s->pool_rows;
-    ext.rope_rows = c.max_position;
     ext.a_elems = sel ? sel->a_elems : 0;
     CUDA_TRY(prof_launch(m, K_EMBED_NORM, 1, 0.0, T * H * 8.0, st, [&] {
       return launch_embed(w.tok_id + t0, Tc, build ? build->x : m->embed, m->attn_norm, H, c.rms_eps, w.r, w.xn,
                           w.ss_e, ext, st);
     }));
     GemmParams base{};
-    base.ext = ext;
     base.M = Tc;
     base.norm_dim = H;
     base.eps = c.rms_eps;

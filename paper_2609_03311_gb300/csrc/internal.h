@@ -29,7 +29,6 @@ struct Extents {
   int64_t rows = 0;        // rows of the chunk's activation buffers (packed tokens)
   int64_t table_rows = 0;  // rows of the table a gather reads (embedding, or a build's input vectors)
   int64_t pool_rows = 0;   // 256-byte rows of the store pool
-  int64_t rope_rows = 0;   // positions of the RoPE table
   int64_t a_elems = 0;     // floats of the key token selection's attention matrices
 };
 
@@ -211,7 +210,6 @@ struct GemmParams {
   int q_cols, k_cols;
   int* err;
   uint64_t timeout_ns;
-  Extents ext;
 };
 cudaError_t gemm_setup();
 // C[M][N] = A[M][K] * B[N][K]^T followed by the epilogue `epi`.

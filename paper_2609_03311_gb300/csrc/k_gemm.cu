@@ -139,10 +139,7 @@ __device__ __forceinline__ void epilogue_prefetch(const GemmParams& p, int mb, i
   if constexpr (EPI == EPI_QKV) {
     if (nb * BN + part * 128 < p.q_cols + p.k_cols)
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int pos = p.tok_pos[min(row0 + i * 4 + (lane >> 3), p.M - 1)];
-        pre.pos[i] = index_ok(p.ext.err, pos, p.ext.rope_rows) ? pos : 0;  // RoPE table row
-      }
+      for (int i = 0; i < 8; ++i) pre.pos[i] = p.tok_pos[min(row0 + i * 4 + (lane >> 3), p.M - 1)];
   }
 }
 
