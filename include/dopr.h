@@ -49,10 +49,17 @@ typedef enum {
     DOPR_ERR_TIMEOUT = 6,       /* a bounded device wait ran out; the result
                                    of that call is invalid, the context is not */
     DOPR_ERR_UNSUPPORTED = 7,   /* a shape this build does not handle         */
-    DOPR_ERR_INTERNAL = 8       /* a checked build (DOPR_CHECKED) met an index
+    DOPR_ERR_INTERNAL = 8,      /* a checked build (DOPR_CHECKED) met an index
                                    outside its buffer and skipped the access:
                                    a library defect; the call's outputs are
                                    invalid, the context is not               */
+    DOPR_ERR_RANGE = 9          /* a value the tensor cores take as an fp16
+                                   operand (normed activations, q/k/v, the
+                                   SwiGLU output, the attention output) or a
+                                   score was not finite or exceeded 65504 in
+                                   magnitude: the inputs leave the range the
+                                   fp16 path computes on; the call's outputs
+                                   are invalid, the context is not           */
 } dopr_status;
 
 /*
@@ -106,8 +113,12 @@ DOPR_API dopr_status dopr_model_create(const dopr_model_config *cfg, dopr_model 
 /* Copy one weight tensor into the model (converted to the library's own
  * device layout).  `src` holds n_elems bf16 values in the layout listed
  * under dopr_weight_kind; src_on_device != 0 means `src` is a device
- * pointer.  Re-putting a weight replaces it.  Synchronous.
- * Errors: INVALID_ARG (kind, layer or n_elems wrong), CUDA. */
+ * pointer.  Re-putting a weight replaces it.  Synchronous.  The
+ * projection matrices (Q, K, V, O, gate, up, down) are held as fp16 for
+ * the tensor cores: a value that is not finite or exceeds 65504 in
+ * magnitude fails the put (the weight is then left as it was).
+ * Errors: INVALID_ARG (kind, layer or n_elems wrong; a projection value
+ * outside fp16's range), CUDA. */
 DOPR_API dopr_status dopr_model_put_weight(dopr_model *model, int32_t kind, int32_t layer, const void *src,
                                   int64_t n_elems, int32_t src_on_device);
 
@@ -240,12 +251,19 @@ DOPR_API int64_t dopr_prefix_bytes(const dopr_model_config *cfg, int32_t m);
  * exactly in its normal range -- with fp32 accumulation, an fp32 residual
  * stream and fp32 norms, softmax and score head.
  * The call is synchronous in both modes: it synchronises `cuda_stream`
- * once after packing (to size the launches) and once at the end, then
- * reports the device error word.  Pairs of one doc_id are grouped so that
- * their prefix is staged once per group; scores do not depend on batch
- * order.  With io_on_device = 1 the inputs are validated on the device and
- * an invalid batch returns its error before any decoder kernel runs.
- * Errors: INVALID_ARG, UNKNOWN_DOC, INCOMPLETE, OUT_OF_MEMORY, CUDA, TIMEOUT.
+ * once after packing (to size the launches) and once after the last
+ * kernel, reads the device error word, and only when it is clear copies
+ * the scores into `scores` (a third synchronisation): a call that fails,
+ * on the host or on the device, writes nothing.  Pairs of one doc_id are
+ * grouped so that their prefix is staged once per group; scores do not
+ * depend on batch order.  With io_on_device = 1 the inputs are validated
+ * on the device and an invalid batch returns its error before any decoder
+ * kernel runs.
+ * Valid range: every fp16 operand must stay within +-65504 (the bf16
+ * inputs are checked at put time; intermediates are checked as they are
+ * written, see DOPR_ERR_RANGE).
+ * Errors: INVALID_ARG, UNKNOWN_DOC, INCOMPLETE, OUT_OF_MEMORY, CUDA, TIMEOUT,
+ * RANGE, INTERNAL (checked builds).
  */
 DOPR_API dopr_status dopr_score(dopr_model *model, dopr_store *store, int32_t n_pairs, const int32_t *q_offsets,
                        const int32_t *q_tokens, const int64_t *doc_ids, float *scores, void *cuda_stream,
@@ -326,6 +344,10 @@ DOPR_API dopr_status dopr_debug_wait_timeout(int32_t timeout_ms);
  *   perm      [n_pairs] int32 DEVICE output: input index of sorted pair s.
  *   tok_off   [n_pairs+1] int32 DEVICE output: first packed token of sorted
  *             pair s (query tokens + the score token per pair).
+ * Validation is dopr_score's: unknown or incomplete documents, decreasing
+ * offsets and m + query length + 1 > max_position (the store's, which
+ * dopr_score requires to equal the model's) fail the call.  The C ABI carries
+ * no buffer sizes: the caller guarantees the extents above.
  * Limits: n_pairs <= 32768 and store max_doc_id < 131072; larger requests
  * return DOPR_ERR_UNSUPPORTED with a message and launch nothing.  The scratch
  * array (about 768 KiB) is held by every GPU that loads the library until the

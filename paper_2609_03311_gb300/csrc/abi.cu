@@ -276,6 +276,10 @@ dopr_status map_device_error(int e) {
   if (e & DEV_ERR_BAD_OFFSETS) return fail(DOPR_ERR_INVALID_ARG, "q_offsets must start at 0 and not decrease");
   if (e & DEV_ERR_POSITION) return fail(DOPR_ERR_INVALID_ARG, "m + query length + 1 exceeds max_position");
   if (e & DEV_ERR_BOUNDS) return fail(DOPR_ERR_INTERNAL, "checked build: an index outside its buffer (access skipped)");
+  if (e & DEV_ERR_RANGE)
+    return fail(DOPR_ERR_RANGE,
+                "an intermediate fp16 operand (normed activations, q/k/v, SwiGLU output, attention output) or a "
+                "score was not finite or exceeded 65504 in magnitude; the call's scores are invalid");
   return DOPR_OK;
 }
 
@@ -321,8 +325,13 @@ void prof_collect(Model* m) {
   p.pending.clear();
 }
 
+// A store serves a model when its per-layer K/V blocks have the model's shape and both
+// bound positions alike (the packer checks m + query length against max_position, and
+// dopr_pack_order_noalloc, which sees only the store, must accept exactly what
+// dopr_score accepts).
 bool same_shape(const dopr_model_config& a, const dopr_model_config& b) {
-  return a.n_layers == b.n_layers && a.n_kv_heads == b.n_kv_heads && a.head_dim == b.head_dim;
+  return a.n_layers == b.n_layers && a.n_kv_heads == b.n_kv_heads && a.head_dim == b.head_dim &&
+         a.max_position == b.max_position;
 }
 
 // Host validation of host-resident inputs (before any launch).
@@ -871,7 +880,7 @@ dopr_status store_mark(Store* s, int32_t slot, int layer, bool present) {
 
 dopr_status check_ready(Model* m, Store* s) {
   if (!m || !s) return fail(DOPR_ERR_INVALID_ARG, "model or store is NULL");
-  if (!same_shape(m->cfg, s->cfg)) return fail(DOPR_ERR_INVALID_ARG, "store shape does not match the model");
+  if (!same_shape(m->cfg, s->cfg)) return fail(DOPR_ERR_INVALID_ARG, "store shape (layers, kv heads, head_dim, max_position) does not match the model");
   const int L = m->cfg.n_layers;
   for (int k = 0; k < kind_count(); ++k)
     for (int l = 0; l < (kind_is_global(k) ? 1 : L); ++l)
@@ -1031,11 +1040,22 @@ dopr_status dopr_model_put_weight(dopr_model* m, int32_t kind, int32_t layer, co
   if (!matrix) {
     CUDA_TRY(cudaMemcpy(dst, src, (size_t)expect * 2, dir));
   } else {
-    // stage, widen bf16 -> fp16 (exact in fp16's normal range), then place
+    // stage, widen bf16 -> fp16 (exact in fp16's normal range), then place; a value
+    // outside fp16's range (or not finite) fails the put and leaves the weight as it was
     void* stage = nullptr;
-    CUDA_TRY(cudaMalloc(&stage, (size_t)expect * 2));
+    const size_t bytes = ((size_t)expect * 2 + 15) & ~(size_t)15;
+    CUDA_TRY(cudaMalloc(&stage, bytes + 16));
+    int* d_range = reinterpret_cast<int*>(static_cast<uint8_t*>(stage) + bytes);
+    int range = 0;
     cudaError_t e = cudaMemcpy(stage, src, (size_t)expect * 2, dir);
-    if (e == cudaSuccess) e = launch_bf16_to_f16(stage, expect, 0);
+    if (e == cudaSuccess) e = cudaMemset(d_range, 0, sizeof(int));
+    if (e == cudaSuccess) e = launch_bf16_to_f16(stage, expect, d_range, 0);
+    if (e == cudaSuccess) e = cudaMemcpy(&range, d_range, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && range) {
+      cudaFree(stage);
+      return fail(DOPR_ERR_INVALID_ARG,
+                  "weight kind %d layer %d: a value is not finite or exceeds the fp16 range (|x| > 65504)", kind, layer);
+    }
     if (e == cudaSuccess) {
       if (kind == DOPR_W_GATE || kind == DOPR_W_UP)  // rows 128b.. go to rows 256b (+128 for up)
         e = cudaMemcpy2D(dst, 256 * H * 2, stage, 128 * H * 2, 128 * H * 2, F / 128, cudaMemcpyDeviceToDevice);
@@ -1433,7 +1453,6 @@ dopr_status dopr_score(dopr_model* m, dopr_store* s, int32_t n, const int32_t* q
   Workspace& w = m->ws;
   const int32_t *dqo = q_offsets, *dqt = q_tokens;
   const int64_t* ddoc = doc_ids;
-  float* dsc = scores;
   if (!io_on_device) {
     if (n > 0 && q_offsets[n] > 0 && !q_tokens) return fail(DOPR_ERR_INVALID_ARG, "q_tokens is NULL");
     STATUS_TRY(validate_host_inputs(m, s, n, q_offsets, q_tokens, doc_ids));
@@ -1445,18 +1464,22 @@ dopr_status dopr_score(dopr_model* m, dopr_store* s, int32_t n, const int32_t* q
     dqo = w.q_off;
     dqt = w.q_tok;
     ddoc = w.doc_ids;
-    dsc = w.scores;
   } else {
     STATUS_TRY(ensure_call_buffers(m, n, 0, 0, s->max_doc_id + 1));
   }
   Plan plan;
   STATUS_TRY(run_packer(m, s, n, dqo, dqt, ddoc, st, plan));
-  STATUS_TRY(run_layers(m, s, plan, dsc, st));
-  if (!io_on_device) CUDA_TRY(cudaMemcpyAsync(scores, w.scores, sizeof(float) * n, cudaMemcpyDeviceToHost, st));
+  // scores land in the workspace and reach the caller only once the device error
+  // word is known to be clear: a failed call writes nothing
+  STATUS_TRY(run_layers(m, s, plan, w.scores, st));
   CUDA_TRY(cudaMemcpyAsync(w.h_err, w.err, sizeof(int), cudaMemcpyDeviceToHost, st));
   CUDA_TRY(cudaStreamSynchronize(st));
   prof_collect(m);
-  return map_device_error(*w.h_err);
+  STATUS_TRY(map_device_error(*w.h_err));
+  CUDA_TRY(cudaMemcpyAsync(scores, w.scores, sizeof(float) * n,
+                           io_on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost, st));
+  CUDA_TRY(cudaStreamSynchronize(st));
+  return DOPR_OK;
 }
 
 dopr_status dopr_debug_pack_plan(dopr_model* m, dopr_store* s, int32_t n, const int32_t* q_offsets,
@@ -1464,7 +1487,7 @@ dopr_status dopr_debug_pack_plan(dopr_model* m, dopr_store* s, int32_t n, const 
                                  int32_t* tok_pos, int32_t* tok_id, int32_t* tok_pair) {
   g_last_error.clear();
   if (!m || !s) return fail(DOPR_ERR_INVALID_ARG, "model or store is NULL");
-  if (!same_shape(m->cfg, s->cfg)) return fail(DOPR_ERR_INVALID_ARG, "store shape does not match the model");
+  if (!same_shape(m->cfg, s->cfg)) return fail(DOPR_ERR_INVALID_ARG, "store shape (layers, kv heads, head_dim, max_position) does not match the model");
   if (n < 0 || !q_offsets || (n > 0 && (!doc_ids || !perm || !tok_off))) return fail(DOPR_ERR_INVALID_ARG, "bad args");
   if (n == 0) {
     tok_off[0] = 0;

@@ -22,7 +22,16 @@ enum : int {
   DEV_ERR_BAD_OFFSETS = 1 << 4,  // q_offsets decreasing / not starting at 0
   DEV_ERR_POSITION = 1 << 5,     // m + query length reaches max_position
   DEV_ERR_BOUNDS = 1 << 6,       // checked build: an index outside its buffer (the access was skipped)
+  DEV_ERR_RANGE = 1 << 7,        // a value written as an fp16 operand (or a score) was not finite or |x| > 65504
 };
+
+// True when x is finite and fits fp16's range (|x| <= 65504, the largest finite
+// fp16); NaN compares false.  Epilogues that write fp16 operands OR the negation
+// into a per-thread flag and report it once per tile (report_range).
+__device__ __forceinline__ bool fp16_ok(float x) { return fabsf(x) <= 65504.f; }
+__device__ __forceinline__ void report_range(int* err, bool bad) {
+  if (__any_sync(0xffffffffu, bad) && (threadIdx.x & 31) == 0 && err) atomicOr(err, DEV_ERR_RANGE);
+}
 
 // Index tests of checked builds (compiled with -DDOPR_CHECKED).  index_ok(err,
 // i, n) is true when 0 <= i < n; otherwise it sets DEV_ERR_BOUNDS in *err and
@@ -293,11 +302,12 @@ __device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 // Two bf16 values (one 32-bit word) -> the same two values as fp16 (exact in
-// fp16's normal range; magnitudes above 65504 saturate).
-__device__ __forceinline__ uint32_t bf16x2_to_f16x2(uint32_t w) {
+// fp16's normal range).  Sets `bad` when either value is not finite or its
+// magnitude exceeds 65504 (the caller rejects the whole conversion).
+__device__ __forceinline__ uint32_t bf16x2_to_f16x2(uint32_t w, bool& bad) {
   const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w));
-  const float lo = fminf(fmaxf(f.x, -65504.f), 65504.f), hi = fminf(fmaxf(f.y, -65504.f), 65504.f);
-  return pack_f16x2(lo, hi);
+  bad |= !(fp16_ok(f.x) && fp16_ok(f.y));
+  return pack_f16x2(f.x, f.y);
 }
 
 __device__ __forceinline__ float warp_sum(float v) {

@@ -221,8 +221,9 @@ cudaError_t launch_gemm(int epi, const CUtensorMap& tmA, const CUtensorMap& tmB,
 // the embedding and the first RMSNorm.
 cudaError_t launch_embed(const int32_t* tok_id, int T, const bf16* embed, const bf16* gain, int H, float eps, float* r,
                          f16* xn, float* ss, const Extents& ext, cudaStream_t st);
-// In place: n bf16 values -> fp16 (saturating at +-65504).
-cudaError_t launch_bf16_to_f16(void* buf, int64_t n, cudaStream_t st);
+// In place: n bf16 values -> fp16; *range |= 1 (device int) when a value is not finite
+// or above 65504 in magnitude.
+cudaError_t launch_bf16_to_f16(void* buf, int64_t n, int* range, cudaStream_t st);
 // Score head over sorted pairs [p_begin, p_end): the score-token row of pair s is
 // r[tok_off[s+1]-1-tok0], or r[s - p_begin] when `compact` is set.
 cudaError_t launch_score(const float* r, int H, const int32_t* tok_off, int tok0, int p_begin, int p_end, int compact,

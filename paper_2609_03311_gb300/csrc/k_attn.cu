@@ -190,9 +190,14 @@ __device__ __forceinline__ void store_tile(const AttnArgs& a, const PairGeom& pg
       const int hh = row % G;
       f16* dst = a.out + static_cast<int64_t>(orow) * a.ld_out + (g * G + hh) * HEAD_DIM + (lane & 3) * 2;
       const float inv = hr ? inv1 : inv0;
+      bool bad = false;
 #pragma unroll
-      for (int dt = 0; dt < 16; ++dt)
-        *reinterpret_cast<uint32_t*>(dst + dt * 8) = pack_f16x2(st.o[dt][2 * hr] * inv, st.o[dt][2 * hr + 1] * inv);
+      for (int dt = 0; dt < 16; ++dt) {
+        const float y0 = st.o[dt][2 * hr] * inv, y1 = st.o[dt][2 * hr + 1] * inv;
+        bad |= !(fp16_ok(y0) && fp16_ok(y1));
+        *reinterpret_cast<uint32_t*>(dst + dt * 8) = pack_f16x2(y0, y1);
+      }
+      if (bad && a.err) atomicOr(a.err, DEV_ERR_RANGE);
     }
   }
 }

@@ -334,14 +334,20 @@ __global__ void __launch_bounds__(THREADS, 1)
       int is = 0, js = 0, nbs = 0;  // S: unit, next block, blocks
       bool s_open = false;          // unit is's Q and region are in hand
       int ip = 0, jp = 0;           // P V: unit, next block
-      uint64_t idle_since = globaltimer_ns();
+      int nk_p = -1;                // key columns of unit ip (read once it is needed)
+      // Idle polls are cheap barrier tests; the error word (a global load) and the clock
+      // are read only every IDLE_CHECK idle polls, so a hand-off is seen within one poll.
+      constexpr uint32_t IDLE_CHECK = 2048;
+      uint32_t idle = 0;
+      uint64_t idle_since = 0;
       bool ok = true;
       while (ip < n_local) {
         bool prog = false;
         // ---- O = P V of unit ip, whose S is complete; P is read from TMEM
         if (ip < is) {
           const int slot = ip & 1;
-          const int n_keys = a.tiles[unit_of(ip) / a.Hkv].n_keys;
+          if (nk_p < 0) nk_p = a.tiles[unit_of(ip) / a.Hkv].n_keys;  // once per unit, not per poll
+          const int n_keys = nk_p;
           const int nbp = (n_keys + KBLK - 1) / KBLK;
           auto p_ready = [&](int j) {
             return mbar_test(bar(BAR_P_FULL + slot * MAX_BLOCKS + j), (ppar >> (slot * MAX_BLOCKS + j)) & 1u);
@@ -369,6 +375,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             for (int j = 0; j < nbp; ++j) ppar ^= 1u << (slot * MAX_BLOCKS + j);  // each block's barrier completed once
             ++ip;
             jp = 0;
+            nk_p = -1;
             prog = true;
           }
         }
@@ -415,11 +422,15 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
         }
         if (prog) {
-          idle_since = globaltimer_ns();
-        } else if ((ld_volatile(a.err) & DEV_ERR_TIMEOUT) || globaltimer_ns() - idle_since > WAIT_TIMEOUT_NS) {
-          atomicOr(a.err, DEV_ERR_TIMEOUT);
-          ok = false;
-          break;
+          idle = 0;
+        } else if (++idle % IDLE_CHECK == 0) {
+          const uint64_t now = globaltimer_ns();
+          if (idle == IDLE_CHECK) idle_since = now;  // the first check of this idle stretch
+          if ((ld_volatile(a.err) & DEV_ERR_TIMEOUT) || now - idle_since > WAIT_TIMEOUT_NS) {
+            atomicOr(a.err, DEV_ERR_TIMEOUT);
+            ok = false;
+            break;
+          }
         }
       }
       // every MMA this thread issued is complete once the drain barrier flips
@@ -510,6 +521,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (!mbar_wait(bar(BAR_O_FULL + slot), par, a.err, WAIT_TIMEOUT_NS)) break;
       tc_fence_after();
       const float inv = sum > 0.f ? 1.f / sum : 0.f;
+      bool bad = false;  // a stored output value not finite or beyond fp16's range
 #pragma unroll 1
       for (int h = 0; h < 2; ++h) {
 #pragma unroll
@@ -525,11 +537,17 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const uint32_t* x = v + 8 * q;
+            float y[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              y[e] = __uint_as_float(x[e]) * inv;
+              bad |= valid && !fp16_ok(y[e]);  // rows past the tile's tokens are not stored
+            }
             uint4 o;
-            o.x = pack_f16x2(__uint_as_float(x[0]) * inv, __uint_as_float(x[1]) * inv);
-            o.y = pack_f16x2(__uint_as_float(x[2]) * inv, __uint_as_float(x[3]) * inv);
-            o.z = pack_f16x2(__uint_as_float(x[4]) * inv, __uint_as_float(x[5]) * inv);
-            o.w = pack_f16x2(__uint_as_float(x[6]) * inv, __uint_as_float(x[7]) * inv);
+            o.x = pack_f16x2(y[0], y[1]);
+            o.y = pack_f16x2(y[2], y[3]);
+            o.z = pack_f16x2(y[4], y[5]);
+            o.w = pack_f16x2(y[6], y[7]);
             const int chunk = c2 * 4 + q;
             *reinterpret_cast<uint4*>(stg + lane * 128 + ((chunk ^ (lane & 7)) << 4)) = o;
           }
@@ -548,6 +566,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         __syncwarp();  // staging reads finish before the next half's writes
       }
+      if (bad) atomicOr(a.err, DEV_ERR_RANGE);
     }
   }
 
@@ -923,6 +942,7 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
       if (!mbar_wait(bar(lt::B_O_FULL), static_cast<uint32_t>(i) & 1u, a.err, WAIT_TIMEOUT_NS)) break;
       tc_fence_after();
       const float inv = sum > 0.f ? 1.f / sum : 0.f;
+      bool bad = false;  // a stored output value not finite or beyond fp16's range
 #pragma unroll 1
       for (int h = 0; h < 2; ++h) {
         uint32_t v2[2][32];
@@ -940,11 +960,17 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const uint32_t* x = v + 8 * q;
+            float y[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              y[e] = __uint_as_float(x[e]) * inv;
+              bad |= valid && !fp16_ok(y[e]);  // rows past the tile's tokens are not stored
+            }
             uint4 o;
-            o.x = pack_f16x2(__uint_as_float(x[0]) * inv, __uint_as_float(x[1]) * inv);
-            o.y = pack_f16x2(__uint_as_float(x[2]) * inv, __uint_as_float(x[3]) * inv);
-            o.z = pack_f16x2(__uint_as_float(x[4]) * inv, __uint_as_float(x[5]) * inv);
-            o.w = pack_f16x2(__uint_as_float(x[6]) * inv, __uint_as_float(x[7]) * inv);
+            o.x = pack_f16x2(y[0], y[1]);
+            o.y = pack_f16x2(y[2], y[3]);
+            o.z = pack_f16x2(y[4], y[5]);
+            o.w = pack_f16x2(y[6], y[7]);
             const int chunk = c2 * 4 + q;
             *reinterpret_cast<uint4*>(stg + lane * 128 + ((chunk ^ (lane & 7)) << 4)) = o;
           }
@@ -963,6 +989,7 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
         }
         __syncwarp();  // staging reads finish before the next half's writes
       }
+      if (bad) atomicOr(a.err, DEV_ERR_RANGE);
     }
   }
 

@@ -147,6 +147,9 @@ template <int EPI>
 __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t taddr, int mb, int nb, int quarter,
                                               int part, int lane, uint32_t* xs, const EpiPre& pre) {
   const int row0 = mb * BM + quarter * 32;  // first row of this warp; lane = row - row0 = TMEM lane
+  bool bad = false;  // a value written as fp16 is not finite or beyond 65504 (reported once per tile)
+  // this lane's row exists (rows past M hold whatever the operand buffers held there; never stored)
+  const bool live = row0 + lane < p.M;
   if constexpr (EPI == EPI_STORE || EPI == EPI_QKV) {
     f16* out = reinterpret_cast<f16*>(p.out);
     const float rs = pre.scale;
@@ -225,6 +228,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
                 const float u = a[k] * inv_i[i] * g1[k], w = b[k] * inv_i[i] * g2[k];
                 y1[k] = u * cosv[k] - w * sinv[k];
                 y2[k] = w * cosv[k] + u * sinv[k];
+                bad |= !(fp16_ok(y1[k]) && fp16_ok(y2[k]));
               }
               f16* orow = out + static_cast<int64_t>(row0 + r) * p.ld_out + hc + c + w4;
               *reinterpret_cast<uint2*>(orow) = make_uint2(pack_f16x2(y1[0], y1[1]), pack_f16x2(y1[2], y1[3]));
@@ -241,8 +245,11 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
           tmem_ld_wait();
 #pragma unroll
           for (int j = 0; j < 32; j += 2) {
-            xs[lane * 33 + j / 2] = pack_f16x2(__uint_as_float(a[j]) * rs, __uint_as_float(a[j + 1]) * rs);
-            xs[lane * 33 + 16 + j / 2] = pack_f16x2(__uint_as_float(b[j]) * rs, __uint_as_float(b[j + 1]) * rs);
+            const float a0 = __uint_as_float(a[j]) * rs, a1 = __uint_as_float(a[j + 1]) * rs;
+            const float b0 = __uint_as_float(b[j]) * rs, b1 = __uint_as_float(b[j + 1]) * rs;
+            bad |= live && !(fp16_ok(a0) && fp16_ok(a1) && fp16_ok(b0) && fp16_ok(b1));
+            xs[lane * 33 + j / 2] = pack_f16x2(a0, a1);
+            xs[lane * 33 + 16 + j / 2] = pack_f16x2(b0, b1);
           }
           __syncwarp();
           store_words_transposed(xs, lane, row0, p.M, [&](int r, int wd) {
@@ -308,9 +315,11 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
           if (p.xn_out) {
             ss[i] += x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w;
             const float sc = prev[i];
+            const float n0 = x.x * g4.x * sc, n1 = x.y * g4.y * sc, n2 = x.z * g4.z * sc, n3 = x.w * g4.w * sc;
+            bad |= !(fp16_ok(n0) && fp16_ok(n1) && fp16_ok(n2) && fp16_ok(n3));
             uint2 o;
-            o.x = pack_f16x2(x.x * g4.x * sc, x.y * g4.y * sc);
-            o.y = pack_f16x2(x.z * g4.z * sc, x.w * g4.w * sc);
+            o.x = pack_f16x2(n0, n1);
+            o.y = pack_f16x2(n2, n3);
             *reinterpret_cast<uint2*>(p.xn_out + static_cast<int64_t>(row0 + r) * p.ld_out + col) = o;
           }
         }
@@ -345,6 +354,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
         for (int j = 0; j < 32; j += 2) {
           const float a0 = silu_f(__uint_as_float(g[j]) * rs) * (__uint_as_float(u[j]) * rs);
           const float a1 = silu_f(__uint_as_float(g[j + 1]) * rs) * (__uint_as_float(u[j + 1]) * rs);
+          bad |= live && !(fp16_ok(a0) && fp16_ok(a1));
           xs[lane * 33 + 16 * half + j / 2] = pack_f16x2(a0, a1);
         }
       }
@@ -355,6 +365,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
       __syncwarp();
     }
   }
+  report_range(p.err, bad);
 }
 
 template <int EPI>

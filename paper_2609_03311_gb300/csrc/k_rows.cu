@@ -43,6 +43,7 @@ __global__ void __launch_bounds__(ROW_WARPS * 32)
   }
   ss = warp_sum(ss);
   const float inv = rsqrtf(ss / static_cast<float>(H) + eps);
+  bool bad = false;
   for (int c = lane * 8; c < H; c += 256) {
     const uint4 w = *reinterpret_cast<const uint4*>(e + c);
     const uint4 gw = *reinterpret_cast<const uint4*>(gain + c);
@@ -52,18 +53,24 @@ __global__ void __launch_bounds__(ROW_WARPS * 32)
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       const float2 a = __bfloat1622float2(w2[k]), b = __bfloat1622float2(g2[k]);
-      o[k] = pack_f16x2(a.x * inv * b.x, a.y * inv * b.y);
+      const float x0 = a.x * inv * b.x, x1 = a.y * inv * b.y;
+      bad |= !(fp16_ok(x0) && fp16_ok(x1));
+      o[k] = pack_f16x2(x0, x1);
     }
     *reinterpret_cast<uint4*>(xr + c) = make_uint4(o[0], o[1], o[2], o[3]);
   }
+  report_range(ext.err, bad);
   if (lane == 0) ss_out[row] = ss;
 }
 
-// In place bf16 -> fp16 over n values (n even), 16 bytes per thread and step.
-__global__ void k_bf16_to_f16(uint32_t* __restrict__ buf, int64_t n_words) {
+// In place bf16 -> fp16 over n values (n even), one 32-bit word per thread and
+// step; *range |= 1 when a value is not finite or outside fp16's range.
+__global__ void k_bf16_to_f16(uint32_t* __restrict__ buf, int64_t n_words, int* range) {
+  bool bad = false;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n_words;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x)
-    buf[i] = bf16x2_to_f16x2(buf[i]);
+    buf[i] = bf16x2_to_f16x2(buf[i], bad);
+  if (bad) atomicOr(range, 1);
 }
 
 // Score head at the score-token row of each sorted pair in [p_begin, p_end):
@@ -95,7 +102,9 @@ __global__ void __launch_bounds__(ROW_WARPS * 32)
   }
   yes = warp_sum(yes);
   no = warp_sum(no);
-  if (lane == 0) scores[perm[s]] = yes - no;
+  const float sc = yes - no;
+  report_range(ext.err, !isfinite(sc));
+  if (lane == 0) scores[perm[s]] = sc;
 }
 
 // MLP scoring head (Sec. 3.2.3): one CTA per pair.  hn = RMSNorm(row) * g in
@@ -148,6 +157,7 @@ __global__ void __launch_bounds__(MLP_THREADS)
   if (threadIdx.x == 0) {
     float sc = b2;
     for (int w = 0; w < MLP_THREADS / 32; ++w) sc += red[w];
+    if (!isfinite(sc) && ext.err) atomicOr(ext.err, DEV_ERR_RANGE);
     scores[perm[s]] = sc;
   }
 }
@@ -243,11 +253,11 @@ cudaError_t launch_embed(const int32_t* tok_id, int T, const bf16* embed, const 
   return cudaGetLastError();
 }
 
-cudaError_t launch_bf16_to_f16(void* buf, int64_t n, cudaStream_t st) {
+cudaError_t launch_bf16_to_f16(void* buf, int64_t n, int* range, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
   const int64_t words = n / 2;
   int blocks = static_cast<int>(std::min<int64_t>((words + 255) / 256, 4096));
-  k_bf16_to_f16<<<blocks, 256, 0, st>>>(static_cast<uint32_t*>(buf), words);
+  k_bf16_to_f16<<<blocks, 256, 0, st>>>(static_cast<uint32_t*>(buf), words, range);
   return cudaGetLastError();
 }
 

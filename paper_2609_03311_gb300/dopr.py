@@ -18,9 +18,9 @@ from . import build as _build
 _LIB = None
 
 (OK, ERR_INVALID_ARG, ERR_UNKNOWN_DOC, ERR_INCOMPLETE, ERR_OUT_OF_MEMORY, ERR_CUDA, ERR_TIMEOUT, ERR_UNSUPPORTED,
- ERR_INTERNAL) = range(9)
+ ERR_INTERNAL, ERR_RANGE) = range(10)
 STATUS_NAMES = ["OK", "INVALID_ARG", "UNKNOWN_DOC", "INCOMPLETE", "OUT_OF_MEMORY", "CUDA", "TIMEOUT", "UNSUPPORTED",
-                "INTERNAL"]
+                "INTERNAL", "RANGE"]
 
 (W_EMBED, W_ATTN_NORM, W_Q, W_K, W_V, W_Q_NORM, W_K_NORM, W_O, W_MLP_NORM, W_GATE, W_UP, W_DOWN, W_FINAL_NORM,
  W_SCORE_HEAD) = range(14)
@@ -178,6 +178,8 @@ class Store:
     def __init__(self, cfg: ModelConfig, max_doc_id: int, pool_bytes: int):
         self.cfg = cfg
         self._h = ctypes.c_void_p()
+        # the library places the store on the calling thread's current device
+        self.device = torch.cuda.current_device() if torch.cuda.is_available() else 0
         _check(load().dopr_store_create(ctypes.byref(cfg), int(max_doc_id), int(pool_bytes), ctypes.byref(self._h)))
 
     def put_layer(self, doc_id: int, layer: int, k: torch.Tensor, v: torch.Tensor):
@@ -324,6 +326,13 @@ def pack_order_noalloc(store: Store, q_offsets: torch.Tensor, doc_ids: torch.Ten
     assert q_offsets.dtype == torch.int32 and doc_ids.dtype == torch.int64
     assert perm.dtype == torch.int32 and tok_off.dtype == torch.int32
     n = q_offsets.numel() - 1
+    # the C ABI takes no buffer sizes: every extent the packer kernels index is checked here
+    if n < 0 or doc_ids.numel() < n or perm.numel() < n or tok_off.numel() < n + 1:
+        raise ValueError(f"pack_order_noalloc: buffers too short for {n} pairs (doc_ids {doc_ids.numel()}, "
+                         f"perm {perm.numel()}, tok_off {tok_off.numel()}; need {n}, {n}, {n + 1})")
+    for name, t in (("q_offsets", q_offsets), ("doc_ids", doc_ids), ("perm", perm), ("tok_off", tok_off)):
+        if not t.is_contiguous() or t.device.index != store.device:
+            raise ValueError(f"pack_order_noalloc: {name} must be contiguous on cuda:{store.device}")
     st = ctypes.c_void_p(stream.cuda_stream if stream is not None else torch.cuda.current_stream().cuda_stream)
     _check(load().dopr_pack_order_noalloc(store._h, n, _ptr(q_offsets), _ptr(doc_ids), _ptr(perm), _ptr(tok_off),
                                           st))

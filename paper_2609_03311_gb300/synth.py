@@ -23,6 +23,7 @@ any tensor can be regenerated alone.
 """
 from __future__ import annotations
 
+import os
 import zlib
 from dataclasses import dataclass, field, replace
 
@@ -122,7 +123,17 @@ def _generator(device, seed: int, *tags) -> torch.Generator:
     return g
 
 
-def _normal_bf16(shape, std, device, seed, *tags) -> torch.Tensor:
+def _normal_bf16(shape, std, device, seed, *tags, portable=False) -> torch.Tensor:
+    if portable:
+        # float64 draws of torch's CPU generator: its double normal path is scalar
+        # Box-Muller on the Mersenne-Twister stream on every host CPU (the float32
+        # path is vectorised differently on x86 and Arm), so after rounding to bf16
+        # the same seed gives the same bytes on either machine
+        g = _generator("cpu", seed, *tags)
+        x = torch.randn(shape, generator=g, dtype=torch.float64)
+        if std != 1.0:
+            x.mul_(std)
+        return x.to(torch.bfloat16).to(device)
     g = _generator(device, seed, *tags)
     x = torch.randn(shape, generator=g, device=device, dtype=torch.float32)
     if std != 1.0:
@@ -130,54 +141,75 @@ def _normal_bf16(shape, std, device, seed, *tags) -> torch.Tensor:
     return x.to(torch.bfloat16)
 
 
-def _gain_bf16(n, norms, device, seed, *tags) -> torch.Tensor:
+def _gain_bf16(n, norms, device, seed, *tags, portable=False) -> torch.Tensor:
     if norms == "ones":
         return torch.ones(n, device=device, dtype=torch.bfloat16)
+    if portable:
+        g = _generator("cpu", seed, *tags)
+        x = 1.0 + 0.1 * torch.randn(n, generator=g, dtype=torch.float64)
+        return x.to(torch.bfloat16).to(device)
     g = _generator(device, seed, *tags)
     x = 1.0 + 0.1 * torch.randn(n, generator=g, device=device, dtype=torch.float32)
     return x.to(torch.bfloat16)
 
 
 def make_weights(shape: ModelShape, seed: int = 0, device="cpu", norms: str = "ones",
-                 std: float = 0.02, zero: tuple = ()) -> dict:
+                 std: float = 0.02, zero: tuple = (), portable: bool = False) -> dict:
     """Random-init bf16 decoder weights.  ``zero`` names tensors to set to 0
-    (used by closed-form checks).  Layout: matrices are [out, in]."""
+    (used by closed-form checks).  Layout: matrices are [out, in].
+
+    ``portable`` draws every tensor from the host generator in float64 (see
+    _normal_bf16), so the bytes are the same on any host and do not depend on
+    the GPU: stored expected values computed on one machine then hold on
+    another.  The tensors are drawn in parallel threads (one sub-stream each)."""
     s = shape
     D, Hq, Hkv, H, F = s.head_dim, s.n_q_heads, s.n_kv_heads, s.hidden, s.ffn
 
     def mat(name, l, rows, cols):
         if name in zero:
-            return torch.zeros(rows, cols, device=device, dtype=torch.bfloat16)
-        return _normal_bf16((rows, cols), std, device, seed, name, l)
+            return lambda: torch.zeros(rows, cols, device=device, dtype=torch.bfloat16)
+        return lambda: _normal_bf16((rows, cols), std, device, seed, name, l, portable=portable)
 
-    w = {
-        "embed": _normal_bf16((s.vocab, H), std, device, seed, "embed"),
-        "final_norm": _gain_bf16(H, norms, device, seed, "final_norm"),
-        "score_head": mat("score_head", 0, 2, H),
+    def gain(n, name, *tags):
+        return lambda: _gain_bf16(n, norms, device, seed, name, *tags, portable=portable)
+
+    jobs = {
+        ("embed",): lambda: _normal_bf16((s.vocab, H), std, device, seed, "embed", portable=portable),
+        ("final_norm",): gain(H, "final_norm"),
+        ("score_head",): mat("score_head", 0, 2, H),
     }
-    per = {k: [] for k in ("attn_norm", "wq", "wk", "wv", "q_norm", "k_norm", "wo",
-                           "mlp_norm", "w_gate", "w_up", "w_down")}
     for l in range(s.n_layers):
-        per["attn_norm"].append(_gain_bf16(H, norms, device, seed, "attn_norm", l))
-        per["wq"].append(mat("wq", l, Hq * D, H))
-        per["wk"].append(mat("wk", l, Hkv * D, H))
-        per["wv"].append(mat("wv", l, Hkv * D, H))
-        per["q_norm"].append(_gain_bf16(D, norms, device, seed, "q_norm", l))
-        per["k_norm"].append(_gain_bf16(D, norms, device, seed, "k_norm", l))
-        per["wo"].append(mat("wo", l, H, Hq * D))
-        per["mlp_norm"].append(_gain_bf16(H, norms, device, seed, "mlp_norm", l))
-        per["w_gate"].append(mat("w_gate", l, F, H))
-        per["w_up"].append(mat("w_up", l, F, H))
-        per["w_down"].append(mat("w_down", l, H, F))
-    w.update(per)
+        jobs[("attn_norm", l)] = gain(H, "attn_norm", l)
+        jobs[("wq", l)] = mat("wq", l, Hq * D, H)
+        jobs[("wk", l)] = mat("wk", l, Hkv * D, H)
+        jobs[("wv", l)] = mat("wv", l, Hkv * D, H)
+        jobs[("q_norm", l)] = gain(D, "q_norm", l)
+        jobs[("k_norm", l)] = gain(D, "k_norm", l)
+        jobs[("wo", l)] = mat("wo", l, H, Hq * D)
+        jobs[("mlp_norm", l)] = gain(H, "mlp_norm", l)
+        jobs[("w_gate", l)] = mat("w_gate", l, F, H)
+        jobs[("w_up", l)] = mat("w_up", l, F, H)
+        jobs[("w_down", l)] = mat("w_down", l, H, F)
+    if portable:
+        from concurrent.futures import ThreadPoolExecutor
+
+        keys = sorted(jobs, key=lambda k: k != ("embed",))  # the largest draw first
+        with ThreadPoolExecutor(max_workers=max(1, min(32, os.cpu_count() or 1))) as ex:
+            done = dict(zip(keys, ex.map(lambda k: jobs[k](), keys)))
+    else:
+        done = {k: f() for k, f in jobs.items()}
+    w = {"embed": done[("embed",)], "final_norm": done[("final_norm",)], "score_head": done[("score_head",)]}
+    for name in ("attn_norm", "wq", "wk", "wv", "q_norm", "k_norm", "wo", "mlp_norm", "w_gate", "w_up", "w_down"):
+        w[name] = [done[(name, l)] for l in range(s.n_layers)]
     return w
 
 
-def make_prefix(shape: ModelShape, m: int, doc: int, seed: int = 0, device="cpu"):
-    """Stored prefix states of one document: K, V bf16 [L, m, Hkv, D], N(0,1)."""
+def make_prefix(shape: ModelShape, m: int, doc: int, seed: int = 0, device="cpu", portable: bool = False):
+    """Stored prefix states of one document: K, V bf16 [L, m, Hkv, D], N(0,1)
+    (``portable`` as in make_weights)."""
     s = shape
-    k = _normal_bf16((s.n_layers, m, s.n_kv_heads, s.head_dim), 1.0, device, seed, "prefix_k", doc)
-    v = _normal_bf16((s.n_layers, m, s.n_kv_heads, s.head_dim), 1.0, device, seed, "prefix_v", doc)
+    k = _normal_bf16((s.n_layers, m, s.n_kv_heads, s.head_dim), 1.0, device, seed, "prefix_k", doc, portable=portable)
+    v = _normal_bf16((s.n_layers, m, s.n_kv_heads, s.head_dim), 1.0, device, seed, "prefix_v", doc, portable=portable)
     return k, v
 
 

@@ -10,6 +10,7 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 from paper_2609_03311_gb300 import dopr, synth
 
 pytestmark = pytest.mark.gpu
@@ -53,7 +54,11 @@ def test_noalloc_matches_regular_packer_on_consecutive_calls(rig):
     for n, seed in ((700, 1), (33, 2), (700, 1), (1, 3)):
         qo, qt, docs = _batch(doc_m, n, seed)
         ref = dopr.pack_plan(model, store, qo, qt, docs)
+        # the oracle's plan (stable sort by document, packed offsets) fixes both
+        want = oracle.pack_plan(qo, qt, docs, [doc_m[int(d)] for d in docs], SHAPE.score_token_id)
         perm, tok_off = _noalloc(store, qo, docs)
+        np.testing.assert_array_equal(perm, want["perm"])
+        np.testing.assert_array_equal(tok_off, want["tok_off"])
         np.testing.assert_array_equal(perm, ref["perm"])
         np.testing.assert_array_equal(tok_off, ref["tok_off"])
 
@@ -74,9 +79,17 @@ def test_noalloc_limits_and_errors(rig):
         dopr.pack_order_noalloc(store, torch.tensor([0, 3], dtype=torch.int32, device="cuda"),
                                 torch.tensor([5], dtype=torch.int64, device="cuda"), out[:1], out[:2])
     assert ei.value.status == dopr.ERR_UNKNOWN_DOC
+    # short caller buffers are refused by the binding before anything is launched
+    qo3 = torch.tensor([0, 1, 2, 3], dtype=torch.int32, device="cuda")
+    d3 = torch.full((3,), 2, dtype=torch.int64, device="cuda")
+    o3 = torch.full((4,), -7, dtype=torch.int32, device="cuda")
+    for args in ((qo3, d3[:2], o3[:3], o3), (qo3, d3, o3[:2], o3), (qo3, d3, o3[:3], o3[:3])):
+        with pytest.raises(ValueError):
+            dopr.pack_order_noalloc(store, *args)
+    assert torch.all(o3 == -7)
     # still correct after the failed calls
     qo2, qt2, docs2 = _batch(doc_m, 50, 4)
-    ref = dopr.pack_plan(model, store, qo2, qt2, docs2)
+    want = oracle.pack_plan(qo2, qt2, docs2, [doc_m[int(d)] for d in docs2], SHAPE.score_token_id)
     perm, tok_off = _noalloc(store, qo2, docs2)
-    np.testing.assert_array_equal(perm, ref["perm"])
-    np.testing.assert_array_equal(tok_off, ref["tok_off"])
+    np.testing.assert_array_equal(perm, want["perm"])
+    np.testing.assert_array_equal(tok_off, want["tok_off"])
