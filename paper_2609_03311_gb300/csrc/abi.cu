@@ -174,13 +174,13 @@ dopr_status build_weight_maps(Model* m) {
   m->tm_qkv.resize(L); m->tm_o.resize(L); m->tm_gu.resize(L); m->tm_down.resize(L);
   for (int l = 0; l < L; ++l) {
     bool ok = make_tmap_16b_2d(&m->tm_qkv[l], m->w_qkv + (size_t)l * m->qkv_dim * H, H, m->qkv_dim, (uint64_t)H * 2,
-                               GEMM_BK, GEMM_BN, true, true) &&
+                               GEMM_BK, GEMM_B_BOX, true, true) &&
               make_tmap_16b_2d(&m->tm_o[l], m->w_o + (size_t)l * H * m->o_dim, m->o_dim, H, (uint64_t)m->o_dim * 2,
-                               GEMM_BK, GEMM_BN, true, true) &&
+                               GEMM_BK, GEMM_B_BOX, true, true) &&
               make_tmap_16b_2d(&m->tm_gu[l], m->w_gu + (size_t)l * 2 * F * H, H, 2 * F, (uint64_t)H * 2, GEMM_BK,
-                               GEMM_BN, true, true) &&
+                               GEMM_B_BOX, true, true) &&
               make_tmap_16b_2d(&m->tm_down[l], m->w_down + (size_t)l * H * F, F, H, (uint64_t)F * 2, GEMM_BK,
-                               GEMM_BN, true, true);
+                               GEMM_B_BOX, true, true);
     if (!ok) return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for layer %d weights", l);
   }
   m->maps_ok = true;
@@ -792,7 +792,7 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
       pd.K = F;
       pd.out = resid;
       pd.ld_out = H;
-      if (!last) {
+      if (!final_layer) {  // a next layer exists: emit its attention norm's operand
         pd.xn_out = w.xn;
         pd.xn_gain = m->attn_norm + (size_t)(l + 1) * H;
         pd.ss_out = w.ss_a;
@@ -1331,7 +1331,12 @@ dopr_status dopr_select_prefix_inputs(dopr_model* m, int32_t n_docs, const int32
   // a store of one empty document gives the attention kernels a valid pool map
   dopr_store* empty = nullptr;
   STATUS_TRY(dopr_store_create(&c, 0, 256, &empty));
-  std::unique_ptr<dopr_store, void (*)(dopr_store*)> hold(empty, [](dopr_store* x) { dopr_store_destroy(x); });
+  // freed on return without touching this thread's error message (dopr_store_destroy clears it)
+  std::unique_ptr<dopr_store, void (*)(dopr_store*)> hold(empty, [](dopr_store* x) {
+    cudaSetDevice(x->device);
+    free_store(x);
+    delete x;
+  });
   dopr_status rs = ensure_call_buffers(m, n_docs, T, 0, 0);
   if (rs != DOPR_OK) return rs;
   std::vector<int32_t> tok_pos(T), tok_pair(T);
@@ -1566,7 +1571,7 @@ dopr_status dopr_debug_gemm(int32_t M, int32_t N, int32_t K, const void* A, cons
   if (gemm_setup() != cudaSuccess) return fail(DOPR_ERR_CUDA, "gemm setup failed");
   CUtensorMap ta, tb;
   if (!make_tmap_16b_2d(&ta, A, K, M, (uint64_t)K * 2, GEMM_BK, GEMM_BM, true, true) ||
-      !make_tmap_16b_2d(&tb, B, K, N, (uint64_t)K * 2, GEMM_BK, GEMM_BN, true, true))
+      !make_tmap_16b_2d(&tb, B, K, N, (uint64_t)K * 2, GEMM_BK, GEMM_B_BOX, true, true))
     return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed (pointers must be 16-byte aligned)");
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
