@@ -183,6 +183,8 @@ bool make_tmap_q_heads(CUtensorMap* map, const void* base, uint64_t cols, uint64
 // GEMM epilogues.
 enum GemmEpi : int { EPI_STORE = 0, EPI_RESID_ADD = 1, EPI_SWIGLU = 2, EPI_QKV = 3 };
 constexpr int GEMM_BM = 128, GEMM_BN = 256, GEMM_BK = 64;
+// Rows of a B (weight) tensor-map box: each CTA of a pair stages 128 of a tile's 256 B rows.
+constexpr int GEMM_B_BOX = 128;
 constexpr int GEMM_SS_PER_TILE = 2;  // partial sums of squares a residual epilogue writes per row and n-tile
 struct GemmParams {
   int M, N, K;

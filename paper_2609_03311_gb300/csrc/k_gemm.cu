@@ -2,21 +2,30 @@
 // the 5th-generation tensor cores: C[M][N] = A[M][K] * B[N][K]^T, fp16
 // operands, fp32 accumulate in tensor memory, fused epilogues.
 //
-// Design (sm_103a, one CTA per SM, persistent):
-//   warp 0      TMA producer: 128x64 A tile + 256x64 B tile per stage, 128-byte
-//               swizzle, 4-stage shared-memory ring guarded by full/empty mbarriers;
-//   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and one
-//               elected thread issues tcgen05.mma (M=128, N=256, K=16) per k-step,
-//               committing stage releases and accumulator-ready barriers;
-//   warps 2..9  epilogue: tcgen05.ld the finished accumulator (one TMEM lane quarter
-//               = 32 rows per warp, one row per thread; two warps per quarter, each
-//               taking half of the tile's 256 columns), apply the epilogue in that
-//               row-per-thread layout, then transpose 32x32-word chunks through
-//               padded shared memory so every global access is a 128-byte row
-//               segment written by 8 consecutive lanes; finally release the
-//               accumulator so the next tile's MMAs overlap the epilogue.
-// Tiles are visited in groups of 16 M-blocks so the weight tiles a wave reads
-// stay in L2 while the activation rows of the group are reused across N.
+// Design (sm_103a, CTA pairs, persistent): a cluster of two CTAs on two SMs
+// computes one 256 x 256 output tile with tcgen05 cta_group::2 MMAs (M = 256,
+// N = 256, K = 16).  Each CTA stages its own 128 rows of A and its own 128 of
+// the tile's 256 B rows per 64-wide k-block (32 KiB a stage, 6-stage ring,
+// 128-byte swizzle); the MMAs read both CTAs' shared memory, so per SM a
+// third less operand data moves into shared memory and out of it into the
+// tensor core per FLOP than with a 128 x 256 tile on one SM.  Roles:
+//   warp 0      (both CTAs) TMA producer; the copies of both CTAs complete on
+//               the leader's full barrier of the stage;
+//   warp 1      allocates 512 TMEM columns in both CTAs (two accumulators of
+//               256 columns); in the leader one thread issues the MMAs and
+//               commits stage releases and accumulator-ready barriers to both
+//               CTAs (multicast);
+//   warps 2..9  (both CTAs) epilogue on the CTA's 128 rows of the tile:
+//               tcgen05.ld the finished accumulator (one TMEM lane quarter =
+//               32 rows per warp, one row per thread; two warps per quarter,
+//               each taking half of the tile's 256 columns), apply the
+//               epilogue in that row-per-thread layout, then transpose 32x32-
+//               word chunks through padded shared memory so every global
+//               access is a 128-byte row segment written by 8 consecutive
+//               lanes; finally tell the leader the accumulator is free, so the
+//               next tile's MMAs overlap the epilogue.
+// Tiles are visited in groups of 8 row blocks (2,048 rows) so the weight tiles
+// a wave reads stay in L2 while the activation rows of the group are reused.
 //
 // Fused epilogues (the decoder's RMSNorms live here, not in separate kernels):
 //   RMSNorm(r) * g = rs * (r (.) g) with rs = rsqrt(mean(r^2) + eps).  The
@@ -29,38 +38,23 @@
 //   q/k gain and rotate-half RoPE at the token's position (pairs i, i+64),
 //   the rotation applied in the transposed layout so RoPE-table reads coalesce.
 //   SwiGLU epilogue: silu(rs * gate) * (rs * up).
+//   Every value written as fp16 is checked against fp16's range (DEV_ERR_RANGE).
 // Every barrier wait is bounded (DEV_ERR_TIMEOUT) and the kernel always drains
-// its own copies and MMAs and frees TMEM before returning.
+// its own MMAs and frees TMEM before returning.
 #include "device_common.cuh"
 #include "internal.h"
 
 namespace dopr {
 namespace {
 
-constexpr int BM = GEMM_BM, BN = GEMM_BN, BK = GEMM_BK;
-constexpr int STAGES = 4;
+constexpr int BM = GEMM_BM, BN = GEMM_BN, BK = GEMM_BK;  // BM: one CTA's rows of a pair tile
+static_assert(GEMM_B_BOX == BM, "each CTA of a pair stages 128 of a tile's 256 B rows");
 constexpr int A_BYTES = BM * BK * 2;  // 16 KiB
-constexpr int B_BYTES = BN * BK * 2;  // 32 KiB
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int TMEM_COLS = 2 * BN;     // two accumulators
 constexpr int THREADS = 320;
 constexpr int EPI_WARPS = 8;
-constexpr int GROUP_M = 16;
 constexpr int XPOSE_WORDS = 32 * 33;  // per epilogue warp: 32 rows x 32 words, padded row stride 33
 constexpr int XPOSE_BYTES = EPI_WARPS * XPOSE_WORDS * 4;
 constexpr int BAR_BYTES = 256;
-constexpr int SMEM_BYTES = 1024 /*alignment slack*/ + STAGES * STAGE_BYTES + XPOSE_BYTES + BAR_BYTES;
-constexpr uint32_t IDESC = umma_idesc_f16(BM, BN);
-
-__device__ __forceinline__ void tile_coords(int t, int m_tiles, int n_tiles, int& mb, int& nb) {
-  const int group = GROUP_M * n_tiles;
-  const int g = t / group;
-  const int first_m = g * GROUP_M;
-  const int gm = min(GROUP_M, m_tiles - first_m);
-  const int r = t - g * group;
-  mb = first_m + r % gm;
-  nb = r / gm;
-}
 
 __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + __expf(-x)); }
 
@@ -368,35 +362,68 @@ __device__ __forceinline__ void epilogue_tile(const GemmParams& p, uint32_t tadd
   report_range(p.err, bad);
 }
 
+// ============================================================================
+// The pair kernel.  Barriers:
+//   full[s]   leader's: armed by the leader for both CTAs' bytes; both CTAs' copies
+//             complete on it (the peer addresses it through the cluster window);
+//   empty[s]  each CTA's: the leader's commit arrives on both (multicast);
+//   tfull[a]  each CTA's: the leader's commit at the end of a tile, multicast;
+//   tempty[a] leader's: all 16 epilogue warps of the pair arrive when TMEM is read.
+constexpr int PAIR_BM = 2 * BM;                 // rows of a pair tile
+constexpr int PAIR_STAGES = 6;
+constexpr int PAIR_B_BYTES = BM * BK * 2;       // this CTA's 128 of the tile's 256 B rows: 16 KiB
+constexpr int PAIR_STAGE_BYTES = A_BYTES + PAIR_B_BYTES;
+constexpr int PAIR_SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + XPOSE_BYTES + BAR_BYTES;
+constexpr int PAIR_GROUP_M = 8;                 // 2,048 rows per L2 group
+constexpr uint32_t PAIR_IDESC = umma_idesc_f16(PAIR_BM, BN);
+// TMEM columns a pair CTA allocates, and accumulators (256 columns each) it cycles through
+constexpr int PAIR_ACCS = 2;
+constexpr uint32_t PAIR_TMEM_COLS = PAIR_ACCS * BN;
+static_assert(PAIR_SMEM_BYTES <= 227 * 1024, "shared memory budget");
+
+__device__ __forceinline__ void pair_tile_coords(int t, int m_tiles, int n_tiles, int& mb, int& nb) {
+  const int group = PAIR_GROUP_M * n_tiles;
+  const int g = t / group;
+  const int first_m = g * PAIR_GROUP_M;
+  const int gm = min(PAIR_GROUP_M, m_tiles - first_m);
+  const int r = t - g * group;
+  mb = first_m + r % gm;
+  nb = r / gm;
+}
+
 template <int EPI>
-__global__ void __launch_bounds__(THREADS, 1)
-    k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmParams p) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
+    k_gemm_pair(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sA = smem_u32(smem);
-  const uint32_t sB = sA + STAGES * A_BYTES;
-  uint32_t* xpose = reinterpret_cast<uint32_t*>(smem + STAGES * STAGE_BYTES);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES + XPOSE_BYTES);
+  const uint32_t sB = sA + PAIR_STAGES * A_BYTES;
+  uint32_t* xpose = reinterpret_cast<uint32_t*>(smem + PAIR_STAGES * PAIR_STAGE_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + PAIR_STAGES * PAIR_STAGE_BYTES + XPOSE_BYTES);
   const uint32_t bar0 = smem_u32(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
-  auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
-  auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
-  auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
-  const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 5);
+  auto empty_bar = [&](int s) { return bar0 + 8u * (PAIR_STAGES + s); };
+  auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * PAIR_STAGES + a); };
+  auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * PAIR_STAGES + 2 + a); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * PAIR_STAGES + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * PAIR_STAGES + 5);
+  static_assert((2 * PAIR_STAGES + 5) * 8 + 4 <= BAR_BYTES, "barrier area");
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m_tiles = (p.M + BM - 1) / BM, n_tiles = p.N / BN, k_blocks = p.K / BK;
-  const int total = m_tiles * n_tiles;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+  const int m_tiles = (p.M + PAIR_BM - 1) / PAIR_BM, n_tiles = p.N / BN, k_blocks = p.K / BK;
+  int total = m_tiles * n_tiles;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < PAIR_STAGES; ++s) {
       mbar_init(full_bar(s), 1);
       mbar_init(empty_bar(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull_bar(a), 1);
-      mbar_init(tempty_bar(a), EPI_WARPS);
+      mbar_init(tempty_bar(a), 2 * EPI_WARPS);
     }
     mbar_init(drain_bar, 1);
     fence_mbar_init();
@@ -404,120 +431,132 @@ __global__ void __launch_bounds__(THREADS, 1)
     tma_prefetch_desc(&tmB);
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_u32(tmem_slot), PAIR_TMEM_COLS);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // both CTAs' barriers exist before either addresses the other's
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  {
+    // the MMAs write both CTAs' TMEM at the leader's address: both allocations must agree
+    uint32_t other;
+    asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(other) : "r"(mapa_shared(smem_u32(tmem_slot), rank ^ 1u)));
+    if (other != tmem_base) {
+      if (threadIdx.x == 0) atomicOr(p.err, DEV_ERR_BOUNDS);
+      total = 0;  // no tile runs
+    }
+  }
 
   if (warp == 0) {
     if (lane == 0) {
-      // ---------------- TMA producer
+      // ---------------- TMA producer (both CTAs): own A rows and own half of B's rows
       int stage = 0;
       uint32_t phase = 0;
-      uint32_t issued = 0, issued_par = 0;  // per stage: ever armed / parity of last arm
       bool ok = true;
-      for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+      for (int t = pair; t < total && ok; t += n_pairs) {
         int mb, nb;
-        tile_coords(t, m_tiles, n_tiles, mb, nb);
+        pair_tile_coords(t, m_tiles, n_tiles, mb, nb);
         for (int kb = 0; kb < k_blocks; ++kb) {
-          if (!mbar_wait(empty_bar(stage), phase ^ 1u, p.err, p.timeout_ns)) {
+          if (!mbar_wait_cluster(empty_bar(stage), phase ^ 1u, p.err, p.timeout_ns)) {
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(full_bar(stage), STAGE_BYTES);
-          tma_load_2d(sA + stage * A_BYTES, &tmA, full_bar(stage), kb * BK, mb * BM);
-          tma_load_2d(sB + stage * B_BYTES, &tmB, full_bar(stage), kb * BK, nb * BN);
-          issued |= 1u << stage;
-          issued_par = (issued_par & ~(1u << stage)) | (phase << stage);
-          if (++stage == STAGES) {
+          if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * PAIR_STAGE_BYTES);
+          const uint32_t fb = mapa_shared(full_bar(stage), 0);
+          tma_load_2d_pair(sA + stage * A_BYTES, &tmA, fb, kb * BK, mb * PAIR_BM + static_cast<int>(rank) * BM);
+          tma_load_2d_pair(sB + stage * PAIR_B_BYTES, &tmB, fb, kb * BK, nb * BN + static_cast<int>(rank) * BM);
+          if (++stage == PAIR_STAGES) {
             stage = 0;
             phase ^= 1u;
           }
         }
       }
       if (!ok) {
-        // Let every copy this thread started land before the CTA can exit.
-        for (int s = 0; s < STAGES; ++s)
-          if (issued & (1u << s)) mbar_wait(full_bar(s), (issued_par >> s) & 1u, p.err, 100000000ull);
+        // copies in flight land within microseconds; give them that long before the
+        // CTA can reach its exit (no barrier to wait on: they count on the leader's)
+        const uint64_t t0 = globaltimer_ns();
+        while (globaltimer_ns() - t0 < 20000ull) {
+        }
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ---------------- MMA issuer
+    if (lane == 0 && leader) {
+      // ---------------- MMA issuer (leader only)
       int stage = 0;
       uint32_t phase = 0;
       int local = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++local) {
-        const int acc = local & 1;
-        const uint32_t acc_phase = (local >> 1) & 1;
-        if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, p.err, p.timeout_ns)) {
+      for (int t = pair; t < total && ok; t += n_pairs, ++local) {
+        const int acc = local % PAIR_ACCS;
+        const uint32_t acc_phase = (local / PAIR_ACCS) & 1;
+        if (!mbar_wait_cluster(tempty_bar(acc), acc_phase ^ 1u, p.err, p.timeout_ns)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
         for (int kb = 0; kb < k_blocks; ++kb) {
-          if (!mbar_wait(full_bar(stage), phase, p.err, p.timeout_ns)) {
+          if (!mbar_wait_cluster(full_bar(stage), phase, p.err, p.timeout_ns)) {
             ok = false;
             break;
           }
           tc_fence_after();
           const uint64_t ad = umma_desc_sw128(sA + stage * A_BYTES);
-          const uint64_t bd = umma_desc_sw128(sB + stage * B_BYTES);
+          const uint64_t bd = umma_desc_sw128(sB + stage * PAIR_B_BYTES);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)  // +32 bytes along K per step, in 16-byte units
-            umma_f16(d_tmem, ad + 2 * k, bd + 2 * k, IDESC, (kb | k) != 0);
-          umma_commit(empty_bar(stage));
-          if (++stage == STAGES) {
+            umma_f16_pair(d_tmem, ad + 2 * k, bd + 2 * k, PAIR_IDESC, (kb | k) != 0);
+          umma_commit_pair_mc(empty_bar(stage), 3);  // both CTAs' stage is free once these MMAs end
+          if (++stage == PAIR_STAGES) {
             stage = 0;
             phase ^= 1u;
           }
         }
-        if (ok) umma_commit(tfull_bar(acc));
+        if (ok) umma_commit_pair_mc(tfull_bar(acc), 3);
       }
       // All MMAs this thread issued are complete once drain_bar flips.
-      umma_commit(drain_bar);
+      umma_commit_pair_mc(drain_bar, 1);
       mbar_wait(drain_bar, 0, p.err, ok ? p.timeout_ns : 100000000ull);
     }
   } else {
-    // ---------------- epilogue warps 2..9 -> TMEM lane quarters 2,3,0,1 (x2), column halves 0/1
+    // ---------------- epilogue warps 2..9 (both CTAs) on this CTA's 128 rows of the tile
     const int quarter = warp & 3;
     const int part = (warp - 2) >> 2;
     uint32_t* xs = xpose + (warp - 2) * XPOSE_WORDS;
     int local = 0;
-    for (int t = blockIdx.x; t < total; t += gridDim.x, ++local) {
-      int mb, nb;
-      tile_coords(t, m_tiles, n_tiles, mb, nb);
-      const int acc = local & 1;
-      const uint32_t acc_phase = (local >> 1) & 1;
+    for (int t = pair; t < total; t += n_pairs, ++local) {
+      int mb2, nb;
+      pair_tile_coords(t, m_tiles, n_tiles, mb2, nb);
+      const int mb = 2 * mb2 + static_cast<int>(rank);  // this CTA's 128-row block
+      const int acc = local % PAIR_ACCS;
+      const uint32_t acc_phase = (local / PAIR_ACCS) & 1;
       EpiPre pre;
       epilogue_prefetch<EPI>(p, mb, nb, quarter, part, lane, pre);
-      if (!mbar_wait(tfull_bar(acc), acc_phase, p.err, p.timeout_ns)) break;
+      if (!mbar_wait_cluster(tfull_bar(acc), acc_phase, p.err, p.timeout_ns)) break;
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
       epilogue_tile<EPI>(p, taddr, mb, nb, quarter, part, lane, xs, pre);
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(tempty_bar(acc));
+      if (lane == 0) mbar_arrive_cluster(mapa_shared(tempty_bar(acc), 0));
     }
   }
 
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // neither CTA leaves while the other may still address its barriers or TMEM
   tc_fence_after();
   if (warp == 1) {
     __syncwarp();
-    tmem_dealloc(tmem_base, TMEM_COLS);
+    tmem_dealloc_pair(tmem_base, PAIR_TMEM_COLS);
   }
 }
 
 template <int EPI>
 cudaError_t set_smem() {
-  return cudaFuncSetAttribute(k_gemm_tc<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  return cudaFuncSetAttribute(k_gemm_pair<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, PAIR_SMEM_BYTES);
 }
 
 }  // namespace
@@ -535,20 +574,22 @@ cudaError_t launch_gemm(int epi, const CUtensorMap& tmA, const CUtensorMap& tmB,
   if (params.M <= 0) return cudaSuccess;
   GemmParams p = params;
   p.timeout_ns = WAIT_TIMEOUT_NS;
-  const int tiles = ((p.M + BM - 1) / BM) * (p.N / BN);
-  const int grid = tiles < num_sms ? tiles : num_sms;
+  // one CTA pair per two SMs (persistent), never more pairs than 256-row tiles
+  const int tiles = ((p.M + PAIR_BM - 1) / PAIR_BM) * (p.N / BN);
+  const int pairs = tiles < num_sms / 2 ? tiles : num_sms / 2;
+  const int grid = 2 * (pairs > 0 ? pairs : 1);
   switch (epi) {
     case EPI_STORE:
-      k_gemm_tc<EPI_STORE><<<grid, THREADS, SMEM_BYTES, st>>>(tmA, tmB, p);
+      k_gemm_pair<EPI_STORE><<<grid, THREADS, PAIR_SMEM_BYTES, st>>>(tmA, tmB, p);
       break;
     case EPI_RESID_ADD:
-      k_gemm_tc<EPI_RESID_ADD><<<grid, THREADS, SMEM_BYTES, st>>>(tmA, tmB, p);
+      k_gemm_pair<EPI_RESID_ADD><<<grid, THREADS, PAIR_SMEM_BYTES, st>>>(tmA, tmB, p);
       break;
     case EPI_SWIGLU:
-      k_gemm_tc<EPI_SWIGLU><<<grid, THREADS, SMEM_BYTES, st>>>(tmA, tmB, p);
+      k_gemm_pair<EPI_SWIGLU><<<grid, THREADS, PAIR_SMEM_BYTES, st>>>(tmA, tmB, p);
       break;
     default:
-      k_gemm_tc<EPI_QKV><<<grid, THREADS, SMEM_BYTES, st>>>(tmA, tmB, p);
+      k_gemm_pair<EPI_QKV><<<grid, THREADS, PAIR_SMEM_BYTES, st>>>(tmA, tmB, p);
       break;
   }
   return cudaGetLastError();
