@@ -57,10 +57,13 @@ def parse_args(argv=None):
                     help="select the workload by configuration number (overrides --workload)")
     ap.add_argument("--queries-per-step", type=int, default=20)
     ap.add_argument("--seed", type=int, default=0)
-    ap.add_argument("--cpu-seconds", type=float, default=15.0, help="bound of the oracle CPU-baseline sample")
+    ap.add_argument("--cpu-seconds", type=float, default=120.0,
+                    help="bound on the oracle time of the CPU-baseline sample (8 length-stratified pairs)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--latency-queries", type=int, default=10)
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the bounded measurement of every configuration after the headline")
     ap.add_argument("--reuse", action="store_true",
                     help="amortised cost under document reuse (T_off, T_full, T_online, Speedup(r)) instead of the bench")
     args = ap.parse_args(argv)
@@ -160,8 +163,11 @@ def slice_pairs(pairs, p0, p1):
 
 
 def oracle_sample(wl, w_host, doc_m, pairs, idx, seed, deadline_s, gen_device):
-    """Score pairs idx[0], idx[1], ... with the oracle until deadline_s of CPU
-    time is used (at least one pair).  Returns (scores dict, seconds, threads)."""
+    """Score pairs idx[0], idx[1], ... with the oracle until deadline_s of oracle
+    time is used (at least one pair).  The prefix states are drawn and copied to
+    the host before the clock starts; only the oracle's scoring is timed.
+    Returns (scores dict, seconds, threads); the scored pairs' token count is
+    in oracle_sample.tokens after the call."""
     import oracle
     from paper_2609_03311_gb300 import synth
 
@@ -169,19 +175,36 @@ def oracle_sample(wl, w_host, doc_m, pairs, idx, seed, deadline_s, gen_device):
     om = oracle.OracleModel(oracle.Shape(s.n_layers, s.hidden, s.n_q_heads, s.n_kv_heads, s.head_dim, s.ffn,
                                          s.vocab, s.rope_theta, s.rms_eps, s.score_token_id), w_host)
     got = {}
-    t0 = time.perf_counter()
+    secs = 0.0
+    oracle_sample.tokens = 0
     for p in idx:
         d = int(pairs["doc_ids"][p])
         m = int(doc_m[d])
-        # the same draw the store received (same seed, same generator device)
+        # the same draw the store received (same seed, same generator device), moved to the host untimed
         k, v = synth.make_prefix(s, m, d, seed=seed, device=gen_device)
+        kv = [(k.cpu(), v.cpu())]
         one = slice_pairs(pairs, p, p + 1)
-        got[int(p)] = float(om.score_pairs(one["q_offsets"], one["q_tokens"], [0], [(k.cpu(), v.cpu())])[0])
-        if time.perf_counter() - t0 >= deadline_s:
+        t0 = time.perf_counter()
+        got[int(p)] = float(om.score_pairs(one["q_offsets"], one["q_tokens"], [0], kv)[0])
+        secs += time.perf_counter() - t0
+        oracle_sample.tokens += len(one["q_tokens"]) + 1
+        if secs >= deadline_s:
             break
-    return got, time.perf_counter() - t0, oracle.num_threads()
+    return got, secs, oracle.num_threads()
 
 
+def stratified_pairs(wl, pairs, n_queries, n):
+    """A length-stratified sample of n pairs from the first n_queries queries'
+    candidate lists: the queries at n evenly spaced quantiles of query length
+    (shortest and longest included), the first candidate of each."""
+    per_q = wl.docs_per_query
+    lens = np.diff(pairs["q_offsets"])[::per_q][:n_queries]
+    order = np.argsort(lens, kind="stable")
+    picks = sorted(set(int(order[round(i * (len(order) - 1) / max(n - 1, 1))]) for i in range(n)))
+    return [q * per_q for q in picks]
+
+
+CPU_SAMPLE_PAIRS = 8  # the oracle's timed sample (the GPU arm's cpu_baseline and the reference arm)
 L2_FLUSH_BYTES = 512 << 20  # four times the 129 MB L2
 
 
@@ -231,14 +254,24 @@ def setup(wl, seed, device, need_host_weights):
         w_host = {k: (v.cpu() if isinstance(v, torch.Tensor) else [t.cpu() for t in v]) for k, v in w.items()}
     del w
     torch.cuda.empty_cache()
+    store, doc_m = make_store(cfg, wl, seed, device)
+    return cfg, model, store, doc_m, w_host
+
+
+def make_store(cfg, wl, seed, device):
+    """The workload's prefix store (every document, drawn on `device`)."""
+    import torch
+
+    from paper_2609_03311_gb300 import dopr, synth
+
     doc_m = synth.doc_prefix_lengths(wl, seed=seed)
     pool = sum(dopr.prefix_bytes(cfg, int(m)) for m in doc_m) + (1 << 20)
     store = dopr.Store(cfg, wl.n_docs - 1, pool)
     for d in range(wl.n_docs):
-        k, v = synth.make_prefix(s, int(doc_m[d]), d, seed=seed, device=device)
+        k, v = synth.make_prefix(wl.model, int(doc_m[d]), d, seed=seed, device=device)
         store.put(d, k, v)
     torch.cuda.synchronize()
-    return cfg, model, store, doc_m, w_host
+    return store, doc_m
 
 
 def gemm_traffic_record():
@@ -253,6 +286,133 @@ def gemm_traffic_record():
     if rec.get("k_gemm_sha256") != hashlib.sha256(src).hexdigest():
         return None
     return rec
+
+
+def kernel_table(prof, steps, peaks):
+    """Per kernel family: launches and ms per step, share of kernel time, achieved
+    TFLOP/s and GB/s on algorithmic work, and the roofline fraction (the slower of
+    FLOPs at the sustained tensor peak and bytes at the HBM peak, over the time)."""
+    tot_ms = sum(v["time_ms"] for v in prof.values()) or 1e-9
+    kernels = {}
+    for name, v in prof.items():
+        if v["launches"] == 0:
+            continue
+        t_s = v["time_ms"] / 1e3
+        ent = {"launches_per_step": v["launches"] / steps, "ms_per_step": v["time_ms"] / steps,
+               "share": v["time_ms"] / tot_ms}
+        if t_s > 0:
+            tf = v["flops"] / t_s / 1e12
+            gbs = v["bytes"] / t_s / 1e9
+            t_roof = max(v["flops"] / (peaks["bf16_tflops_sustained"] * 1e12), v["bytes"] / (peaks["hbm_gbs"] * 1e9))
+            ent.update({"tflops": tf, "gbs": gbs, "roofline_frac": t_roof / t_s,
+                        "gbs_frac_of_nominal_hbm": gbs / NOMINAL_HBM_GBS})
+        kernels[name] = ent
+    return kernels
+
+
+# Queries per step of each configuration's measurement in the default run (the headline's
+# 20; 32 for the launch-bound 2-layer model; 10 for the long 4B queries; 2 for the 512-token
+# uncompressed documents), and the bounded step counts it uses.
+CONFIG_QUERIES = {"0": 32, "1": 20, "2": 10, "3": 20, "4": 2}
+CONFIG_WARMUP, CONFIG_STEPS = 2, 3
+
+
+def time_workload(model, store, wl, pairs, Q, steps, warmup, dev, gpu_index):
+    """Steps of Q queries' candidate lists through dopr_score with device-resident inputs
+    (L2 flushed between steps when the streamed weights fit in it); CUDA-event time,
+    clocks sampled meanwhile, per-kernel accounting."""
+    import torch
+
+    from paper_2609_03311_gb300 import dopr
+
+    per_q = wl.docs_per_query
+    n_batches = max(1, wl.n_queries // Q)
+    batches = []
+    for b in range(n_batches):
+        sl = slice_pairs(pairs, b * Q * per_q, (b + 1) * Q * per_q)
+        batches.append((torch.tensor(sl["q_offsets"], device=dev), torch.tensor(sl["q_tokens"], device=dev),
+                        torch.tensor(sl["doc_ids"], device=dev)))
+    for i in range(warmup):
+        dopr.score(model, store, *batches[i % n_batches])
+    stream_bytes = streamed_bytes_per_step(wl)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev) if stream_bytes < L2_FLUSH_BYTES else None
+    stream = torch.cuda.current_stream(dev)
+    torch.cuda.synchronize()
+    dopr.profile_enable(model, True)
+    clocks = ClockSampler(gpu_index)
+    clocks.start()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * steps)]
+    n_pairs = 0
+    for i in range(steps):
+        if flush is not None:
+            flush.zero_()
+        b = batches[(warmup + i) % n_batches]
+        ev[2 * i].record(stream)
+        dopr.score(model, store, *b)
+        ev[2 * i + 1].record(stream)
+        n_pairs += b[2].numel()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    prof = dopr.profile_read(model)
+    dopr.profile_enable(model, False)
+    step_ms = [ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(steps)]
+    total_ms = sum(step_ms) if flush is not None else ev[0].elapsed_time(ev[-1])
+    peaks = measured_peaks()
+    kernels = kernel_table(prof, steps, peaks)
+    gemm = [f for f in ("gemm_qkv", "gemm_o", "gemm_gate_up", "gemm_down") if f in prof]
+    g_ms = sum(prof[f]["time_ms"] for f in gemm)
+    g_tf = sum(prof[f]["flops"] for f in gemm) / (g_ms / 1e3) / 1e12 if g_ms > 0 else None
+    return {"workload": wl.name, "pairs_per_s": n_pairs / (total_ms / 1e3), "ms_per_step": statistics.mean(step_ms),
+            "p50_batch_ms": statistics.median(step_ms), "pairs_per_step": Q * per_q, "steps": steps,
+            "warmup": warmup, "clocks": clk,
+            "roofline_frac": {k: round(v["roofline_frac"], 4) for k, v in kernels.items() if "roofline_frac" in v},
+            "share": {k: round(v["share"], 4) for k, v in kernels.items()},
+            "gemm_tflops": g_tf,
+            "gemm_frac_of_sustained": g_tf / peaks["bf16_tflops_sustained"] if g_tf else None,
+            "l2": "flushed between steps" if flush is not None else "inputs larger than L2"}
+
+
+def run_configs(args, dev, gpu_index, headline, model8=None, cfg8=None):
+    """Every configuration once after the headline, with bounded step counts: pairs/s,
+    clocks and per-kernel roofline fractions; for the uncompressed arm (4) also the
+    speed-up of DoPR (m = 64: the headline's pairs) over it and the doc-side K/V ratio.
+    `model8`, the headline's Qwen3-8B model when it is one, serves configurations 3 and
+    4 and is closed here."""
+    import torch
+
+    from paper_2609_03311_gb300 import dopr, synth
+
+    out = {}
+    for key in ("3", "4", "2", "1", "0"):  # the 8B arms first, while the headline's model is resident
+        wl = synth.WORKLOADS[CONFIG_WORKLOADS[key]]
+        t0 = time.perf_counter()
+        if model8 is not None and wl.model.name == "qwen3-8b":
+            model, own = model8, False
+            store, _ = make_store(cfg8, wl, args.seed, dev)
+        else:
+            if model8 is not None:  # the 8B arms are done: free the headline's model
+                model8.close()
+                model8 = None
+                torch.cuda.empty_cache()
+            _, model, store, _, _ = setup(wl, args.seed, dev, False)
+            own = True
+        pairs = build_pairs(wl, args.seed)
+        r = time_workload(model, store, wl, pairs, min(CONFIG_QUERIES[key], wl.n_queries), CONFIG_STEPS,
+                          CONFIG_WARMUP, dev, gpu_index)
+        r["setup_and_run_s"] = round(time.perf_counter() - t0, 1)
+        store.close()
+        if own:
+            model.close()
+        torch.cuda.empty_cache()
+        out[key] = r
+    if headline.get("workload") == "qwen3-8b-m64":
+        c8 = dopr.make_config(synth.MODELS["qwen3-8b"])
+        out["4"]["dopr_m64_pairs_per_s"] = headline["value"]
+        out["4"]["speedup_dopr_over_uncompressed"] = headline["value"] / out["4"]["pairs_per_s"]
+        out["4"]["doc_kv_bytes_ratio"] = dopr.prefix_bytes(c8, 512) / dopr.prefix_bytes(c8, 64)
+    if model8 is not None:
+        model8.close()
+    return out
 
 
 # ------------------------------------------------------------------ arms
@@ -392,32 +552,26 @@ def run_dopr(args, rank, world, local_rank, dist):
                 "algorithmic_flops_per_launch": g_flops / max(g_launch, 1),
                 "algorithmic_bytes_per_launch": g_bytes / max(g_launch, 1),
                 "share_of_step": g_ms / tot_ms}
-    kernels = {}
-    for name, v in prof.items():
-        if v["launches"] == 0:
-            continue
-        t_s = v["time_ms"] / 1e3
-        ent = {"launches_per_step": v["launches"] / args.steps, "ms_per_step": v["time_ms"] / args.steps,
-               "share": v["time_ms"] / tot_ms}
-        if t_s > 0:
-            tf = v["flops"] / t_s / 1e12
-            gbs = v["bytes"] / t_s / 1e9
-            t_roof = max(v["flops"] / (peaks["bf16_tflops_sustained"] * 1e12), v["bytes"] / (peaks["hbm_gbs"] * 1e9))
-            ent.update({"tflops": tf, "gbs": gbs, "roofline_frac": t_roof / t_s,
-                        "gbs_frac_of_nominal_hbm": gbs / NOMINAL_HBM_GBS})
-        kernels[name] = ent
+    kernels = kernel_table(prof, args.steps, peaks)
     gpu_launches = sum(v["launches"] for v in prof.values())
 
     # ---------------- CPU baseline: the oracle on a bounded sample, rank 0, N = 1
     cpu = parity = None
     if want_cpu:
-        b, scores = outs[0]
-        gpu_scores = scores.cpu().numpy()
-        idx = [b["first_pair"] + j for j in range(len(b["doc_ids"]))]
+        # the oracle on a length-stratified sample of the workload's first batch (the same
+        # pairs as the reference arm), compared with the GPU scores of that batch
+        b0 = batches[0]
+        gpu_scores = step_dev(b0).cpu().numpy()
+        idx = stratified_pairs(wl, pairs, Q, CPU_SAMPLE_PAIRS)
         got, secs, threads = oracle_sample(wl, w_host, doc_m, pairs, idx, args.seed, args.cpu_seconds, dev)
+        toks = oracle_sample.tokens
+        lens = [int(pairs["q_offsets"][p + 1] - pairs["q_offsets"][p]) for p in got]
         cpu = {"value": len(got) / secs, "unit": "pairs/s", "cores": threads, "kind": "oracle",
-               "sample": f"{len(got)} pair(s) of the first timed batch, fp64 C oracle, {secs:.1f} s"}
-        diffs = [abs(float(gpu_scores[p - b["first_pair"]]) - s) for p, s in got.items()]
+               "tokens_per_s": toks / secs,
+               "sample": f"{len(got)} pair(s), one per query at evenly spaced length quantiles of the first "
+                         f"batch (query lengths {lens}), fp64 C oracle, {secs:.1f} s of scoring (prefix draws "
+                         f"and host copies untimed)"}
+        diffs = [abs(float(gpu_scores[p - b0["first_pair"]]) - s) for p, s in got.items()]
         parity = {"pairs": len(diffs), "max_abs_diff": max(diffs), "tolerance": 3e-2,
                   "oracle_scores": [round(s, 5) for s in got.values()]}
 
@@ -444,6 +598,16 @@ def run_dopr(args, rank, world, local_rank, dist):
                         "p90_ms": lat_sorted[int(0.9 * (len(lat_sorted) - 1))] if lat_sorted else None},
             "kernels": kernels, "parity": parity,
         }
+        if not args.no_configs and world == 1:
+            # every configuration, bounded, after the headline (its store freed; its model
+            # reused by the other Qwen3-8B arms, else freed too)
+            store.close()
+            reuse = wl.model.name == "qwen3-8b"
+            if not reuse:
+                model.close()
+            torch.cuda.empty_cache()
+            line["configs"] = run_configs(args, dev, local_rank, {"workload": wl.name, "value": value},
+                                          model if reuse else None, cfg)
         print(json.dumps(line))
 
 
@@ -549,14 +713,17 @@ def run_reference(args, rank, world):
     doc_m = synth.doc_prefix_lengths(wl, seed=args.seed)
     pairs = build_pairs(wl, args.seed)
     n_total = args.warmup + args.steps
-    budget = args.cpu_seconds
+    # one pair per step, cycling through the GPU arm's length-stratified sample
+    sample = stratified_pairs(wl, pairs, min(args.queries_per_step, wl.n_queries), CPU_SAMPLE_PAIRS)
     for i in range(args.warmup):
-        oracle_sample(wl, w_host, doc_m, pairs, [i], args.seed, 0.0, dev)
-    done, secs, threads = 0, 0.0, 1
+        oracle_sample(wl, w_host, doc_m, pairs, [sample[i % len(sample)]], args.seed, 0.0, dev)
+    done, secs, toks, threads = 0, 0.0, 0, 1
     for i in range(args.steps):
-        got, s, threads = oracle_sample(wl, w_host, doc_m, pairs, [args.warmup + i], args.seed, budget, dev)
+        got, t, threads = oracle_sample(wl, w_host, doc_m, pairs, [sample[(args.warmup + i) % len(sample)]],
+                                        args.seed, 0.0, dev)
         done += len(got)
-        secs += s
+        secs += t
+        toks += oracle_sample.tokens
     value = done / secs
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "pairs/s", "n_gpus": world,
@@ -565,7 +732,10 @@ def run_reference(args, rank, world):
         "data": "synthetic: seeded random-init bf16 weights, N(0,1) prefix K/V, uniform token ids",
         "config": {"workload": wl.name, "pairs_per_step": 1, "steps_total": n_total},
         "cpu_baseline": {"value": value, "unit": "pairs/s", "cores": threads, "kind": "oracle",
-                         "sample": f"{done} pair(s), one per step, fp64 C oracle"},
+                         "tokens_per_s": toks / secs,
+                         "sample": f"{done} pair(s), one per step, cycling through {len(sample)} pairs at evenly "
+                                   f"spaced query-length quantiles of the first batch; fp64 C oracle, scoring "
+                                   f"timed alone"},
         "e2e": {"value": value, "unit": "pairs/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
 
