@@ -403,11 +403,11 @@ struct AttnPlanner {
   std::vector<AttnItem> litems;
 
   // The sorted pairs [pb, pe) of one document (token offsets `to`, t0 the chunk's first token).
-  // Each tile takes up to TT consecutive tokens (at most ATTN_TC_MAX_SEGS pairs).  Its own keys
-  // are the run of packed tokens from the first token of its first pair to its last token, so
-  // one 64-row copy loads 64 of them whatever pairs they belong to.  It is a tensor-core tile
-  // when its key columns fit ATTN_TC_MAX_KEYS -- the tile is cut where the next token would
-  // overflow -- and a long tile, with no key limit, when not even its first token fits.
+  // Each tile takes up to TT consecutive tokens (at most ATTN_TC_MAX_SEGS pairs).  It is a
+  // tensor-core tile when its key columns fit ATTN_TC_MAX_KEYS -- the tile is cut where the
+  // next token would overflow -- and a long tile, with no key limit, when not even its first
+  // token fits.  Both kernels compute a row identically, so which one a row lands in does not
+  // change its result.
   void add(const int32_t* to, int32_t t0, int32_t pb, int32_t pe, int32_t slot, int32_t m, int64_t pool_base) {
     auto c16 = [](int x) { return (x + 15) & ~15; };
     const int pre64 = ((m + 63) / 64) * 64;
@@ -424,14 +424,16 @@ struct AttnPlanner {
     while (tok < end) {
       while (to[pf + 1] - t0 <= tok) ++pf;
       // the tokens [tok, tok + n) a tile takes, and its key columns
-      const int32_t run0 = to[pf] - t0;  // first token of the tile's first pair: the own-key run starts here
       auto grow = [&](bool limit_keys, int32_t& keys) {
-        int32_t n = 0, pp = pf;
+        int32_t n = 0, closed = 0, pp = pf;
         keys = 0;
         while (n < TT && tok + n < end) {
           const int32_t t = tok + n;
-          while (to[pp + 1] - t0 <= t) ++pp;
-          const int32_t k = pre64 + c16(t - run0 + 1);
+          while (to[pp + 1] - t0 <= t) {  // pair pp lies wholly in the tile: its full segment
+            closed += c16(to[pp + 1] - to[pp]);
+            ++pp;
+          }
+          const int32_t k = pre64 + closed + c16(t - (to[pp] - t0) + 1);
           if ((limit_keys && k > ATTN_TC_MAX_KEYS) || pp - pf >= ATTN_TC_MAX_SEGS) break;
           keys = k;
           ++n;
@@ -615,14 +617,17 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
     const double attn_flops_last = 4.0 * HEAD_DIM * Hq * last_keys;
     const double attn_bytes_last = np * 2.0 * Hq * HEAD_DIM * 2 + T * 2.0 * Hkv * HEAD_DIM * 2 +
                                    prefix_rows * Hkv * 2 * HEAD_DIM * 2;
-    // this chunk's packed QKV buffer as TMA maps for the tensor-core attention: one box per
-    // Q tile (both halves of the group's G heads over 128 / G rows), one per 64-key block
+    // this chunk's packed QKV buffer as TMA maps for the tensor-core attention:
+    // Q boxes of 128 / G rows of the group's G heads, own-key boxes of 16, 32 and 64 rows
     const int TT = attn_tc_rows_per_head(Hq / Hkv);
-    CUtensorMap tm_q{}, tm_kv{};
+    CUtensorMap tm_q{}, tm_kv{}, tm_kv32{}, tm_kv64{};
     const int n_tiles = plan.chunk_tile[ci + 1] - plan.chunk_tile[ci];
     const int n_ltiles = plan.chunk_ltile[ci + 1] - plan.chunk_ltile[ci];
-    if (n_tiles + n_ltiles > 0 && !(make_tmap_attn_q(&tm_q, w.qkv, m->qkv_dim, Tc, TT, Hq / Hkv) &&
-                                    make_tmap_attn_kv(&tm_kv, w.qkv, m->qkv_dim, Tc)))
+    if (n_tiles + n_ltiles > 0 &&
+        !(make_tmap_q_heads(&tm_q, w.qkv, m->qkv_dim, Tc, TT, Hq / Hkv) &&
+          make_tmap_16b_2d(&tm_kv, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, 16, true, true) &&
+          make_tmap_16b_2d(&tm_kv32, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, 32, true, true) &&
+          make_tmap_16b_2d(&tm_kv64, w.qkv, m->qkv_dim, Tc, (uint64_t)m->qkv_dim * 2, 64, 64, true, true)))
       return fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for the QKV buffer");
     AttnTcArgs ta{};
     ta.tiles = w.tiles + plan.chunk_tile[ci];
@@ -733,11 +738,11 @@ dopr_status run_layers(Model* m, Store* s, const Plan& plan, float* d_scores, cu
                              cudaError_t e = cudaSuccess;
                              if (!last && ta.n_units > 0) {
                                ta.layer = l;
-                               e = launch_attention_tc(tm_q, tm_kv, s->tm_pool3, ta, sms, st);
+                               e = launch_attention_tc(tm_q, tm_kv, tm_kv32, tm_kv64, s->tm_pool, ta, sms, st);
                              }
                              if (e == cudaSuccess && !last && tl.n_units > 0) {
                                tl.layer = l;
-                               e = launch_attention_tc_long(tm_q, tm_kv, s->tm_pool3, tl, sms, st);
+                               e = launch_attention_tc_long(tm_q, tm_kv, tm_kv32, tm_kv64, s->tm_pool, tl, sms, st);
                              }
                              if (e == cudaSuccess && aa.n_items > 0) e = launch_attention(s->tm_pool, aa, st);
                              return e;
@@ -903,48 +908,21 @@ bool make_tmap_16b_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_
   return r == CUDA_SUCCESS;
 }
 
-namespace {
-bool encode_16b(CUtensorMap* map, const void* base, int rank, const cuuint64_t* dims, const cuuint64_t* strides,
-                const cuuint32_t* box) {
+// The Q columns of a packed QKV buffer [rows][cols] as a 3-D tensor: 128 elements of a head
+// (innermost), rows, heads (256 bytes apart); the box takes 64 elements of box_heads heads over
+// box_rows rows, stored head after head (fp16, 128-byte swizzle).
+bool make_tmap_q_heads(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows,
+                       uint32_t box_heads) {
   auto fn = encode_fn();
   if (!fn) return false;
-  cuuint32_t estr[5] = {1, 1, 1, 1, 1};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, rank, const_cast<void*>(base), dims, strides, box, estr,
+  cuuint64_t dims[3] = {128, rows, cols / 128};
+  cuuint64_t strides[2] = {cols * 2, 256};
+  cuuint32_t box[3] = {64, box_rows, box_heads};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
-}
-}  // namespace
-
-// The q heads of a packed QKV buffer [rows][cols] as a 4-D tensor: 64 elements (innermost),
-// rows, heads (256 bytes apart), the head's two 64-element halves (128 bytes apart).  A box of
-// 64 x box_rows x box_heads x 2 lands as [half][head][row][64]: both halves of the G q heads of
-// one kv group over box_rows rows, each half one 128-byte-swizzled K-major operand.
-bool make_tmap_attn_q(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows,
-                      uint32_t box_heads) {
-  const cuuint64_t dims[4] = {64, rows, cols / 128, 2};
-  const cuuint64_t strides[3] = {cols * 2, 256, 128};
-  const cuuint32_t box[4] = {64, box_rows, box_heads, 2};
-  return encode_16b(map, base, 4, dims, strides, box);
-}
-
-// One head of a packed QKV buffer as a 4-D tensor: 64 elements, rows, the two halves,
-// heads.  A box of 64 x 64 x 2 x 1 lands as [half][row][64]: 64 keys (or values) of one
-// head, both halves, in one copy.
-bool make_tmap_attn_kv(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows) {
-  const cuuint64_t dims[4] = {64, rows, 2, cols / 128};
-  const cuuint64_t strides[3] = {cols * 2, 128, 256};
-  const cuuint32_t box[4] = {64, 64, 2, 1};
-  return encode_16b(map, base, 4, dims, strides, box);
-}
-
-// The store pool (rows of 128 fp16) as a 3-D tensor: 64 elements, rows, the two halves.
-// A box of 64 x 64 x 2 lands as [half][row][64].
-bool make_tmap_pool3(CUtensorMap* map, const void* base, uint64_t rows) {
-  const cuuint64_t dims[3] = {64, rows, 2};
-  const cuuint64_t strides[2] = {HEAD_DIM * 2, 128};
-  const cuuint32_t box[3] = {64, 64, 2};
-  return encode_16b(map, base, 3, dims, strides, box);
 }
 
 }  // namespace dopr
@@ -1155,9 +1133,8 @@ dopr_status dopr_store_create(const dopr_model_config* cfg, int64_t max_doc_id, 
       guard(fail(DOPR_ERR_CUDA, "store initialisation failed"));
   }
   if (st == DOPR_OK &&
-      !(make_tmap_16b_2d(&s->tm_pool, s->pool, HEAD_DIM, std::max<int64_t>(s->pool_rows, 1), HEAD_DIM * 2, 64, 64,
-                         true, true) &&
-        make_tmap_pool3(&s->tm_pool3, s->pool, std::max<int64_t>(s->pool_rows, 1))))
+      !make_tmap_16b_2d(&s->tm_pool, s->pool, HEAD_DIM, std::max<int64_t>(s->pool_rows, 1), HEAD_DIM * 2, 64, 64, true,
+                        true))
     guard(fail(DOPR_ERR_CUDA, "cuTensorMapEncodeTiled failed for the store pool"));
   if (st != DOPR_OK) {
     free_store(s);

@@ -41,13 +41,12 @@ struct AttnItem {
 
 // Tensor-core attention (k_attn_tc.cu).  A tile is up to 128 / G consecutive
 // packed tokens of pairs of one document; its keys are the prefix (ceil64(m)
-// columns) then the contiguous run of packed tokens from the first token of the
-// first pair it touches to the tile's last token (padded to a multiple of 16
-// columns; a row sees its own pair's part of the run, up to itself).  A tile keeps
-// within ATTN_TC_MAX_KEYS columns (k_attn_tc) unless its first token alone needs
-// more (a long tile, k_attn_tc_long, no key limit).  The mma.sync kernel
-// (k_attn.cu) takes the last layer's score-token rows, and every row when 128 / G
-// gives no tile shape.
+// columns) then one segment per pair it touches, from the pair's first token to
+// the tile's last, each padded to a multiple of 16 columns.  A tile keeps within
+// ATTN_TC_MAX_KEYS columns (k_attn_tc) unless its first token alone needs more
+// (a long tile, k_attn_tc_long, no key limit).  The mma.sync kernel (k_attn.cu)
+// takes the last layer's score-token rows, and every row when 128 / G gives no
+// tile shape.
 constexpr int ATTN_TC_MAX_KEYS = 256;
 constexpr int ATTN_TC_MAX_SEGS = 16;  // own segments are >= 16 columns each
 struct __align__(16) AttnTile {
@@ -56,12 +55,10 @@ struct __align__(16) AttnTile {
   int32_t n_tok;       // tokens in the tile (<= 128 / G)
   int32_t m;           // the document's prefix length
   int32_t n_keys;      // key columns (multiple of 16, <= ATTN_TC_MAX_KEYS)
-  int32_t n_seg;       // pairs the tile touches, in token order
+  int32_t n_seg;       // own segments, one per pair the tile touches, in token order
   int32_t pad;
-  // pair s: it starts at token tok_begin + (int16_t)(seg[s] & 0xffff) (<= 0 for a pair
-  // begun before the tile) and has seg[s] >> 16 tokens up to the tile's end; the own-key
-  // run starts at pair 0's first token, so token t sits in key column
-  // ceil64(m) + t - (tok_begin + start of pair 0)
+  // segment s: the pair starts at token tok_begin + (int16_t)(seg[s] & 0xffff) (<= 0 for
+  // a pair begun before the tile) and has seg[s] >> 16 tokens up to the tile's end
   int32_t seg[ATTN_TC_MAX_SEGS];
 };
 
@@ -83,8 +80,7 @@ struct Store {
   std::vector<uint8_t> slot_ok;
   int32_t n_slots = 0;
   int32_t max_m = 0;
-  CUtensorMap tm_pool{};   // 2-D: 64-column x 64-row boxes (the mma.sync attention)
-  CUtensorMap tm_pool3{};  // 3-D: both 64-column halves of 64 rows in one box (the tensor-core attention)
+  CUtensorMap tm_pool{};
   bool tm_pool_ok = false;
 };
 
@@ -181,10 +177,8 @@ struct Model {
 // 2-D map over 16-bit elements (fp16 when `half` is set, else bf16).
 bool make_tmap_16b_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
                       uint32_t box_cols, uint32_t box_rows, bool swizzle128, bool half);
-bool make_tmap_attn_q(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows,
-                      uint32_t box_heads);
-bool make_tmap_attn_kv(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows);
-bool make_tmap_pool3(CUtensorMap* map, const void* base, uint64_t rows);
+bool make_tmap_q_heads(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows,
+                       uint32_t box_heads);
 
 // GEMM epilogues.
 enum GemmEpi : int { EPI_STORE = 0, EPI_RESID_ADD = 1, EPI_SWIGLU = 2, EPI_QKV = 3 };
@@ -285,15 +279,16 @@ struct AttnTcArgs {
 // Q rows per head in a 128-row tile; 0 when the group size does not divide 128 into boxes of >= 8 rows.
 inline int attn_tc_rows_per_head(int G) { return (G >= 1 && G <= 16 && 128 % G == 0) ? 128 / G : 0; }
 cudaError_t attn_tc_setup();
-// tm_q: the chunk's packed QKV buffer as a 4-D map (make_tmap_attn_q): one box is both 64-column
-// halves of the G q heads of a kv group over 128 / G rows; tm_kv: the same buffer as a 4-D map
-// (make_tmap_attn_kv): one box is both halves of one head over 64 rows; tm_pool3: the store pool
-// (make_tmap_pool3): one box is both halves of 64 rows (all fp16, 128-byte swizzle).
-cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool3,
-                                const AttnTcArgs& a, int num_sms, cudaStream_t st);
+// tm_q: the Q heads of the chunk's packed QKV buffer as a 3-D map (make_tmap_q_heads), box 64
+// columns x (128 / G) rows x G heads; tm_kv, tm_kv32, tm_kv64: the same buffer, boxes 64 x 16,
+// 64 x 32 and 64 x 64; tm_pool: the store pool, box 64 x 64 (all fp16, 128-byte swizzle).
+cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv32,
+                                const CUtensorMap& tm_kv64, const CUtensorMap& tm_pool, const AttnTcArgs& a,
+                                int num_sms, cudaStream_t st);
 // Tiles with more than ATTN_TC_MAX_KEYS key columns (same maps and arguments).
-cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool3,
-                                     const AttnTcArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv32,
+                                     const CUtensorMap& tm_kv64, const CUtensorMap& tm_pool, const AttnTcArgs& a,
+                                     int num_sms, cudaStream_t st);
 
 // Packer.
 struct PackArgs {

@@ -5,34 +5,36 @@
 //
 // Work unit = (tile, kv head g).  A tile holds up to TT = 128 / G consecutive
 // packed tokens of pairs that share one document; its 128 rows are the G q
-// heads of group g of those tokens, head-major (row = hh * TT + token).  Its key
-// columns are the document's prefix (columns [0, ceil64(m))) followed by the
-// run of packed tokens from the first token of the tile's first pair to the
-// tile's last token; a row sees the prefix and its own pair's part of the run
-// up to itself.  The host keeps every tile within 256 key columns.  Every TMA
-// copy moves both 64-column halves of its rows at once: one copy per Q tile
-// (the group's G heads), one per 64-key K or V block, prefix or own keys -- the
-// issuing thread, not bandwidth, paced the pipeline when tiles took a dozen
-// small copies each.
+// heads of group g of those tokens, head-major (row = hh * TT + token), so each
+// q head's rows arrive as one TMA box of the packed QKV buffer.  Its key
+// columns are the document's prefix (columns [0, ceil64(m))) followed, for each
+// pair the tile touches, by that pair's own keys from its first token up to the
+// tile's last token, each pair's segment starting on a 16-column boundary: a row
+// then meets its keys at the same positions of the same 16-key MMA steps
+// whatever other pairs share its tile.  The host keeps every tile within 256
+// key columns.
 //
 // Persistent CTAs, one per SM, warp-specialised:
 //   warp 0    TMA producer: the Q tile (two stages), the tile's key blocks of
 //             64 columns into a K ring (five stages) and a V ring (three) --
-//             prefix blocks from the store pool, own-key blocks from the
-//             packed QKV buffer (rows past the chunk read as zeros);
+//             prefix blocks from the store pool in 64-row boxes, own-key
+//             segments from the packed QKV buffer in the largest of 64-, 32-
+//             or 16-row boxes that stays inside one pair's visible tokens;
 //   warp 1    MMA issuer: S = Q K^T into the unit's TMEM region (fp32, up to
-//             256 columns, one N = 64 MMA per block and 16-element step), then
-//             O = P V block by block with P read from TMEM and V from shared
-//             memory as an MN-major operand, into the region's upper 128
-//             columns (over S blocks 2 and 3, when the unit has them, once the
-//             softmax has read them); S of the next unit goes in before P V of
-//             this one;
+//             256 columns; one MMA per 16-element step spans every key block
+//             held in consecutive ring stages), then O = P V block by block
+//             with P read from TMEM and V from shared memory as an MN-major
+//             operand, into the region's upper 128 columns (over S blocks 2
+//             and 3, when the unit has them, once the softmax has read them);
+//             S of the next unit goes in before P V of this one;
 //   warps 2-9 two softmax/epilogue warpgroups taking alternate units, one
 //             thread per tile row (its TMEM lane): an exact two-pass softmax
 //             over the row's S (the maximum over the visible keys, then exp2
 //             and fixed-shape 16-key sums added in key order), P written as
 //             fp16 into TMEM over S columns already read, and after the last
 //             P V step O / sum as fp16, staged per warp for whole-line stores.
+// The exact maximum, the in-order sum and the aligned own segments make every
+// row's result independent of how the batch was cut into tiles.
 // Every wait is bounded; a CTA that gives up lets its copies and MMAs land and
 // frees its TMEM before it exits.
 #include <limits.h>
@@ -46,12 +48,14 @@ namespace {
 
 constexpr int TILE_M = 128;
 constexpr int KBLK = 64;  // key columns per block
+constexpr int GROUP_ROWS = 16;
 constexpr int NSLOT = 2;  // tiles in flight: one softmax warpgroup and one TMEM region each
 constexpr int Q_STAGES = 2, K_STAGES = 5, V_STAGES = 3;
 constexpr int Q_HALF = TILE_M * 128;    // 128 rows x 64 16-bit elements
 constexpr int Q_BYTES = 2 * Q_HALF;     // 32 KB
 constexpr int KV_HALF = KBLK * 128;     // 64 rows x 64 elements
 constexpr int KV_BYTES = 2 * KV_HALF;   // 16 KB
+constexpr int GROUP_BYTES = 2 * GROUP_ROWS * 128;
 constexpr int EP_WARP_BYTES = 32 * 128;  // one warp's 32 rows x 64 fp16 columns of O on the way out
 constexpr int THREADS = 64 + NSLOT * 128;
 constexpr int MAX_BLOCKS = ATTN_TC_MAX_KEYS / KBLK;  // 4
@@ -60,8 +64,10 @@ constexpr int MAX_BLOCKS = ATTN_TC_MAX_KEYS / KBLK;  // 4
 // S blocks 2 and 3 when the unit has them.
 constexpr uint32_t TMEM_COLS = 512, SLOT_COLS = 256, O_COL = 128;
 
-// Shared memory.  Every stage keeps its two 64-column halves together
-// ([half][rows][128 B], the layout one TMA copy of both halves writes).
+// Shared memory.  The K ring is half-major ([half][stage][64 rows][128 B]): the
+// rows of consecutive stages follow one another, so the blocks of a unit that
+// sit in consecutive stages are one K-major operand for a single wide S MMA.
+// Q and V stages keep their two 64-column halves together.
 constexpr int OFF_Q = 0;
 constexpr int OFF_K = OFF_Q + Q_STAGES * Q_BYTES;
 constexpr int OFF_V = OFF_K + K_STAGES * KV_BYTES;
@@ -80,7 +86,6 @@ constexpr int SMEM_BYTES = 1024 + OFF_BAR + N_BARS * 8 + 16;
 static_assert(SMEM_BYTES <= 227 * 1024, "shared memory budget");
 
 constexpr uint32_t IDESC_O = umma_idesc_f16_bmn(TILE_M, HEAD_DIM);
-constexpr uint32_t IDESC_S = umma_idesc_f16(TILE_M, KBLK);  // S of one 64-key block
 
 struct Ring {
   int stage = 0;
@@ -167,6 +172,7 @@ __device__ __forceinline__ float exp_pack(uint32_t (&v)[32], uint32_t mask, floa
 
 __global__ void __launch_bounds__(THREADS, 1)
     k_attn_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
+              const __grid_constant__ CUtensorMap tm_kv32, const __grid_constant__ CUtensorMap tm_kv64,
               const __grid_constant__ CUtensorMap tm_pool, AttnTcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -205,6 +211,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     fence_mbar_init();
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_kv);
+    tma_prefetch_desc(&tm_kv32);
+    tma_prefetch_desc(&tm_kv64);
     tma_prefetch_desc(&tm_pool);
   }
   if (warp == 1) {
@@ -231,8 +239,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       auto issue_q = [&](int tok_begin, int g) -> bool {
         if (!mbar_wait(bar(BAR_Q_EMPTY + rq.stage), rq.phase ^ 1u, a.err, WAIT_TIMEOUT_NS)) return false;
         arm(BAR_Q_FULL + rq.stage, rq.phase, Q_BYTES);
-        // one box: both halves of the TT rows of each of the group's G heads
-        tma_load_4d(sQ + rq.stage * Q_BYTES, &tm_q, bar(BAR_Q_FULL + rq.stage), 0, tok_begin, g * G, 0);
+        for (int h = 0; h < 2; ++h)  // one box per 64-column half: TT rows of each of the group's G heads
+          tma_load_3d(sQ + rq.stage * Q_BYTES + h * Q_HALF, &tm_q, bar(BAR_Q_FULL + rq.stage), h * 64, tok_begin,
+                      g * G);
         rq.next(Q_STAGES);
         return true;
       };
@@ -240,24 +249,59 @@ __global__ void __launch_bounds__(THREADS, 1)
         Ring& r = kv ? rv : rk;
         const int full0 = kv ? BAR_V_FULL : BAR_K_FULL, empty0 = kv ? BAR_V_EMPTY : BAR_K_EMPTY;
         const uint32_t ring = kv ? sV : sK;
-        const int m = tp->m, pre64 = ceil64(m);
-        const int nb = (tp->n_keys + KBLK - 1) / KBLK;
+        const int m = tp->m, n_keys = tp->n_keys, tok_begin = tp->tok_begin;
+        const int pre64 = ceil64(m);
+        const int nb = (n_keys + KBLK - 1) / KBLK;
         const int pool_row = static_cast<int>(tp->pool_base + ((static_cast<int64_t>(a.layer) * 2 + kv) * a.Hkv + g) * m);
-        const int run0 = tp->tok_begin + seg_start(tp->seg[0]);  // the own-key run's first token
-        const int head = a.Hq + kv * a.Hkv + g;
+        const int col0 = (a.Hq + kv * a.Hkv + g) * HEAD_DIM;
         if (kCheckedBuild) {  // report only: the tensor maps bound every copy themselves
-          index_ok(a.ext.err, run0, a.ext.rows);
-          index_ok(a.ext.err, tp->tok_begin + tp->n_tok - 1, a.ext.rows);
+          index_ok(a.ext.err, tok_begin + seg_start(tp->seg[0]), a.ext.rows);
+          index_ok(a.ext.err, tok_begin + tp->n_tok - 1, a.ext.rows);
           if (m > 0) index_ok(a.ext.err, pool_row + m - 1, a.ext.pool_rows);
         }
+        int si = 0, k = 0, key = pre64;  // own-key cursor: segment, row within it, key column
+        int sv = tp->seg[0];
         for (int j = 0; j < nb; ++j) {
           if (!mbar_wait(bar(empty0 + r.stage), r.phase ^ 1u, a.err, WAIT_TIMEOUT_NS)) return false;
-          const uint32_t dst = ring + r.stage * KV_BYTES, fb = bar(full0 + r.stage);
-          arm(full0 + r.stage, r.phase, KV_BYTES);
-          if (j * KBLK < pre64)  // prefix rows (past m they are masked)
-            tma_load_3d(dst, &tm_pool, fb, 0, pool_row + j * KBLK, 0);
-          else  // 64 tokens of the own-key run (past the tile's tokens they are masked)
-            tma_load_4d(dst, &tm_kv, fb, 0, run0 + j * KBLK - pre64, 0, head);
+          // half h of the stage: K halves lie K_STAGES * 8 KB apart (see OFF_K), V halves 8 KB apart
+          const uint32_t dst = kv ? ring + r.stage * KV_BYTES : ring + r.stage * KV_HALF;
+          const uint32_t hstride = kv ? KV_HALF : K_STAGES * KV_HALF;
+          const uint32_t fb = bar(full0 + r.stage);
+          if (j * KBLK < pre64) {
+            arm(full0 + r.stage, r.phase, KV_BYTES);
+            for (int h = 0; h < 2; ++h) tma_load_2d(dst + h * hstride, &tm_pool, fb, h * 64, pool_row + j * KBLK);
+          } else {
+            const int groups = min(KBLK, n_keys - j * KBLK) / GROUP_ROWS;
+            arm(full0 + r.stage, r.phase, groups * GROUP_BYTES);
+            if (groups * GROUP_ROWS == KBLK && key == j * KBLK && k + KBLK <= seg_len(sv)) {
+              // the whole block is 64 consecutive tokens of one pair: one 64-row box per half
+              for (int h = 0; h < 2; ++h)
+                tma_load_2d(dst + h * hstride, &tm_kv64, fb, col0 + h * 64, tok_begin + seg_start(sv) + k);
+              key += KBLK;
+              k += KBLK;
+              if (k >= seg_len(sv) && si + 1 < ATTN_TC_MAX_SEGS) {
+                k = 0;
+                sv = tp->seg[++si];
+              }
+            } else {
+              for (int q = 0; q < groups;) {
+                const int off = key - j * KBLK;  // 0, 16, 32, 48 when the plan is consistent
+                // two groups at once when both are 16 consecutive visible tokens of this pair
+                const int n = (q + 2 <= groups && k + 2 * GROUP_ROWS <= seg_len(sv)) ? 2 : 1;
+                if (off >= 0 && off + n * GROUP_ROWS <= KBLK)  // otherwise skipped and the wait times out
+                  for (int h = 0; h < 2; ++h)
+                    tma_load_2d(dst + off * 128 + h * hstride, n == 2 ? &tm_kv32 : &tm_kv, fb, col0 + h * 64,
+                                tok_begin + seg_start(sv) + k);
+                key += n * GROUP_ROWS;
+                k += n * GROUP_ROWS;
+                q += n;
+                if (k >= seg_len(sv) && si + 1 < ATTN_TC_MAX_SEGS) {
+                  k = 0;
+                  sv = tp->seg[++si];
+                }
+              }
+            }
+          }
           r.next(kv ? V_STAGES : K_STAGES);
         }
         return true;
@@ -347,18 +391,26 @@ __global__ void __launch_bounds__(THREADS, 1)
             tc_fence_after();
             prog = true;
           }
-          while (s_open && js < nbs && mbar_test(bar(BAR_K_FULL + rk.stage), rk.phase)) {
-            // S of key block js: one N = 64 MMA per 16-element step of the head dimension
+          while (s_open && js < nbs) {
+            // the unit's next blocks that sit in consecutive ring stages form one B operand of
+            // 64 * run rows: one N = 64 * run MMA per 16-element step once all of them are in
+            const int run = min(nbs - js, K_STAGES - rk.stage);
+            bool landed = true;
+            for (int t = 0; t < run && landed; ++t) landed = mbar_test(bar(BAR_K_FULL + rk.stage + t), rk.phase);
+            if (!landed) break;
             tc_fence_after();
             const uint64_t qd = umma_desc_sw128(sQ + rq.stage * Q_BYTES);
-            const uint64_t kd = umma_desc_sw128(sK + rk.stage * KV_BYTES);
+            const uint64_t kd = umma_desc_sw128(sK + rk.stage * KV_HALF);
+            const uint32_t idesc = umma_idesc_f16(TILE_M, run * KBLK);
 #pragma unroll
-            for (int ks = 0; ks < HEAD_DIM / 16; ++ks)  // 16 elements = 32 bytes per step; halves 16 KB / 8 KB apart
+            for (int ks = 0; ks < HEAD_DIM / 16; ++ks)  // 16 elements = 32 bytes per step; Q halves 16 KB apart
               umma_f16(tmem + slot * SLOT_COLS + js * KBLK, qd + ((ks >> 2) * Q_HALF + (ks & 3) * 32) / 16,
-                       kd + ((ks >> 2) * KV_HALF + (ks & 3) * 32) / 16, IDESC_S, ks > 0);
-            umma_commit(bar(BAR_K_EMPTY + rk.stage));
-            rk.next(K_STAGES);
-            ++js;
+                       kd + ((ks >> 2) * K_STAGES * KV_HALF + (ks & 3) * 32) / 16, idesc, ks > 0);
+            for (int t = 0; t < run; ++t) {
+              umma_commit(bar(BAR_K_EMPTY + rk.stage));
+              rk.next(K_STAGES);
+            }
+            js += run;
             prog = true;
           }
           if (s_open && js == nbs) {
@@ -409,15 +461,16 @@ __global__ void __launch_bounds__(THREADS, 1)
       // the tile's tokens see the prefix only; nothing of theirs is stored.
       int olo = INT_MAX, ohi = -1;
       if (valid) {
-        const int st0 = seg_start(tp->seg[0]);  // the own-key run starts at token st0 of the tile
+        int seg = pre64;
         for (int si = 0; si < n_seg; ++si) {
           const int sv = tp->seg[si];
           const int st = seg_start(sv), len = seg_len(sv);
-          if (jj < st + len) {  // this row's pair: its tokens st .. jj are columns pre64 + (t - st0)
-            olo = pre64 + (st - st0);
-            ohi = pre64 + (jj - st0);
+          if (jj < st + len) {
+            olo = seg;
+            ohi = seg + (jj - st);
             break;
           }
+          seg += ceil16(len);
         }
       }
       const int wlo = __reduce_min_sync(0xffffffffu, olo);
@@ -542,7 +595,7 @@ constexpr int THREADS = 64 + 128;
 // TMEM: O at [0, 128), S buffer b at S_COL + CH b, P stage s (64 keys as fp16) at P_COL + 32 s
 constexpr uint32_t O_COL = 0, S_COL = 128, P_COL = 384;
 constexpr int OFF_Q = 0;
-constexpr int OFF_K = OFF_Q + Q_STAGES * Q_BYTES;  // stages [half][64 rows], as in the short kernel
+constexpr int OFF_K = OFF_Q + Q_STAGES * Q_BYTES;  // half-major, as in the short kernel
 constexpr int OFF_V = OFF_K + K_STAGES * KV_BYTES;
 constexpr int OFF_EP = OFF_V + V_STAGES * KV_BYTES;
 constexpr int OFF_BAR = OFF_EP + 4 * EP_WARP_BYTES;
@@ -560,6 +613,7 @@ static_assert(P_COL + 32 * P_STAGES <= TMEM_COLS, "P ring inside the allocation"
 
 __global__ void __launch_bounds__(lt::THREADS, 1)
     k_attn_tc_long(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
+                   const __grid_constant__ CUtensorMap tm_kv32, const __grid_constant__ CUtensorMap tm_kv64,
                    const __grid_constant__ CUtensorMap tm_pool, AttnTcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -602,6 +656,8 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
     fence_mbar_init();
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_kv);
+    tma_prefetch_desc(&tm_kv32);
+    tma_prefetch_desc(&tm_kv64);
     tma_prefetch_desc(&tm_pool);
   }
   if (warp == 1) {
@@ -623,36 +679,65 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
         armed |= 1u << b;
         armed_par = (armed_par & ~(1u << b)) | (par << b);
       };
-      // where one tile's K or V blocks come from: block j < ceil64(m) / 64 is prefix rows of
-      // the pool, the rest 64 tokens each of the own-key run
+      // a block stream of one tile's K or V rows: blocks must be issued in order 0, 1, ...
       struct Stream {
-        int kv, pre64, pool_row, run0, head;
+        int kv, si, k, sv, pool_row, col0;
       };
       auto start = [&](const AttnTile* tp, int g, int kv) {
         Stream st;
         st.kv = kv;
-        st.pre64 = ceil64(tp->m);
+        st.si = 0;
+        st.k = 0;
+        st.sv = tp->seg[0];
         st.pool_row = static_cast<int>(tp->pool_base + ((static_cast<int64_t>(a.layer) * 2 + kv) * a.Hkv + g) * tp->m);
-        st.run0 = tp->tok_begin + seg_start(tp->seg[0]);
-        st.head = a.Hq + kv * a.Hkv + g;
+        st.col0 = (a.Hq + kv * a.Hkv + g) * HEAD_DIM;
         if (kCheckedBuild) {  // report only: the tensor maps bound every copy themselves
-          index_ok(a.ext.err, st.run0, a.ext.rows);
+          index_ok(a.ext.err, tp->tok_begin + seg_start(tp->seg[0]), a.ext.rows);
           index_ok(a.ext.err, tp->tok_begin + tp->n_tok - 1, a.ext.rows);
           if (tp->m > 0) index_ok(a.ext.err, st.pool_row + tp->m - 1, a.ext.pool_rows);
         }
         return st;
       };
-      auto issue_block = [&](Stream& st, int j) -> bool {
+      auto issue_block = [&](const AttnTile* tp, Stream& st, int j) -> bool {
         Ring& r = st.kv ? rv : rk;
         const int stages = st.kv ? lt::V_STAGES : lt::K_STAGES;
         const int full0 = st.kv ? lt::B_V_FULL : lt::B_K_FULL, empty0 = st.kv ? lt::B_V_EMPTY : lt::B_K_EMPTY;
         if (!mbar_wait(bar(empty0 + r.stage), r.phase ^ 1u, a.err, WAIT_TIMEOUT_NS)) return false;
-        const uint32_t dst = (st.kv ? sV : sK) + r.stage * KV_BYTES, fb = bar(full0 + r.stage);
-        arm(full0 + r.stage, r.phase, KV_BYTES);
-        if (j * KBLK < st.pre64)
-          tma_load_3d(dst, &tm_pool, fb, 0, st.pool_row + j * KBLK, 0);
-        else
-          tma_load_4d(dst, &tm_kv, fb, 0, st.run0 + j * KBLK - st.pre64, 0, st.head);
+        // half h of the stage: K halves lie K_STAGES * 8 KB apart (half-major K ring), V halves 8 KB apart
+        const uint32_t dst = st.kv ? sV + r.stage * KV_BYTES : sK + r.stage * KV_HALF;
+        const uint32_t hstride = st.kv ? KV_HALF : lt::K_STAGES * KV_HALF;
+        const uint32_t fb = bar(full0 + r.stage);
+        if (j * KBLK < ceil64(tp->m)) {
+          arm(full0 + r.stage, r.phase, KV_BYTES);
+          for (int h = 0; h < 2; ++h) tma_load_2d(dst + h * hstride, &tm_pool, fb, h * 64, st.pool_row + j * KBLK);
+        } else {
+          const int groups = min(KBLK, tp->n_keys - j * KBLK) / GROUP_ROWS;
+          arm(full0 + r.stage, r.phase, groups * GROUP_BYTES);
+          if (groups * GROUP_ROWS == KBLK && st.k + KBLK <= seg_len(st.sv)) {
+            // the whole block is 64 consecutive tokens of one pair: one 64-row box per half
+            for (int h = 0; h < 2; ++h)
+              tma_load_2d(dst + h * hstride, &tm_kv64, fb, st.col0 + h * 64, tp->tok_begin + seg_start(st.sv) + st.k);
+            st.k += KBLK;
+            if (st.k >= seg_len(st.sv) && st.si + 1 < ATTN_TC_MAX_SEGS) {
+              st.k = 0;
+              st.sv = tp->seg[++st.si];
+            }
+          } else {
+            for (int q = 0; q < groups;) {
+              // two groups at once when both are 16 consecutive visible tokens of this pair
+              const int n = (q + 2 <= groups && st.k + 2 * GROUP_ROWS <= seg_len(st.sv)) ? 2 : 1;
+              for (int h = 0; h < 2; ++h)
+                tma_load_2d(dst + q * GROUP_ROWS * 128 + h * hstride, n == 2 ? &tm_kv32 : &tm_kv, fb,
+                            st.col0 + h * 64, tp->tok_begin + seg_start(st.sv) + st.k);
+              st.k += n * GROUP_ROWS;
+              q += n;
+              if (st.k >= seg_len(st.sv) && st.si + 1 < ATTN_TC_MAX_SEGS) {
+                st.k = 0;
+                st.sv = tp->seg[++st.si];
+              }
+            }
+          }
+        }
         r.next(stages);
         return true;
       };
@@ -668,13 +753,16 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
           break;
         }
         arm(lt::B_Q_FULL + rq.stage, rq.phase, Q_BYTES);
-        tma_load_4d(sQ + rq.stage * Q_BYTES, &tm_q, bar(lt::B_Q_FULL + rq.stage), 0, tp->tok_begin, g * G, 0);
+        for (int h = 0; h < 2; ++h)
+          tma_load_3d(sQ + rq.stage * Q_BYTES + h * Q_HALF, &tm_q, bar(lt::B_Q_FULL + rq.stage), h * 64,
+                      tp->tok_begin, g * G);
         rq.next(lt::Q_STAGES);
-        Stream ks = start(tp, g, 0), vs = start(tp, g, 1);
-        for (int j = 0; j < nb && ok; ++j) ok = issue_block(ks, j);  // pass A
-        for (int c = 0; c * 2 < nb && ok; ++c) {                      // pass B, chunk by chunk
-          for (int j = 2 * c; j < min(nb, 2 * c + 2) && ok; ++j) ok = issue_block(ks, j);
-          for (int j = 2 * c; j < min(nb, 2 * c + 2) && ok; ++j) ok = issue_block(vs, j);
+        Stream ka = start(tp, g, 0);
+        for (int j = 0; j < nb && ok; ++j) ok = issue_block(tp, ka, j);
+        Stream kb = start(tp, g, 0), vb = start(tp, g, 1);
+        for (int c = 0; c * 2 < nb && ok; ++c) {
+          for (int j = 2 * c; j < min(nb, 2 * c + 2) && ok; ++j) ok = issue_block(tp, kb, j);
+          for (int j = 2 * c; j < min(nb, 2 * c + 2) && ok; ++j) ok = issue_block(tp, vb, j);
         }
       }
       if (!ok) {
@@ -695,17 +783,24 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
         if (!wait(lt::B_S_FREE + buf, ((cc >> 1) & 1u) ^ 1u)) return false;
         tc_fence_after();
         const uint64_t qd = umma_desc_sw128(sQ + rq.stage * Q_BYTES);
-        for (int j = 2 * c; j < min(nb, 2 * c + 2); ++j) {
-          // S of block j: one N = 64 MMA per 16-element step of the head dimension
-          if (!wait(lt::B_K_FULL + rk.stage, rk.phase)) return false;
+        const int je = min(nb, 2 * c + 2);
+        for (int j = 2 * c; j < je;) {
+          // the chunk's blocks in consecutive ring stages: one N = 64 * run MMA per step
+          const int run = min(je - j, lt::K_STAGES - rk.stage);
+          for (int t = 0; t < run; ++t)
+            if (!wait(lt::B_K_FULL + rk.stage + t, rk.phase)) return false;
           tc_fence_after();
-          const uint64_t kd = umma_desc_sw128(sK + rk.stage * KV_BYTES);
+          const uint64_t kd = umma_desc_sw128(sK + rk.stage * KV_HALF);
+          const uint32_t idesc = umma_idesc_f16(TILE_M, run * KBLK);
 #pragma unroll
           for (int ks = 0; ks < HEAD_DIM / 16; ++ks)
             umma_f16(tmem + lt::S_COL + lt::CH * buf + (j - 2 * c) * KBLK, qd + ((ks >> 2) * Q_HALF + (ks & 3) * 32) / 16,
-                     kd + ((ks >> 2) * KV_HALF + (ks & 3) * 32) / 16, IDESC_S, ks > 0);
-          umma_commit(bar(lt::B_K_EMPTY + rk.stage));
-          rk.next(lt::K_STAGES);
+                     kd + ((ks >> 2) * lt::K_STAGES * KV_HALF + (ks & 3) * 32) / 16, idesc, ks > 0);
+          for (int t = 0; t < run; ++t) {
+            umma_commit(bar(lt::B_K_EMPTY + rk.stage));
+            rk.next(lt::K_STAGES);
+          }
+          j += run;
         }
         umma_commit(bar(lt::B_S_FULL + buf));
         ++cc;
@@ -765,15 +860,16 @@ __global__ void __launch_bounds__(lt::THREADS, 1)
       const bool valid = jj < n_tok;
       int olo = INT_MAX, ohi = -1;
       if (valid) {
-        const int st0 = seg_start(tp->seg[0]);  // the own-key run starts at token st0 of the tile
+        int seg = pre64;
         for (int si = 0; si < n_seg; ++si) {
           const int sv = tp->seg[si];
           const int st = seg_start(sv), len = seg_len(sv);
-          if (jj < st + len) {  // this row's pair: its tokens st .. jj are columns pre64 + (t - st0)
-            olo = pre64 + (st - st0);
-            ohi = pre64 + (jj - st0);
+          if (jj < st + len) {
+            olo = seg;
+            ohi = seg + (jj - st);
             break;
           }
+          seg += ceil16(len);
         }
       }
       // every 32-column chunk of S is read and put through the mask: a chunk no
@@ -914,19 +1010,21 @@ cudaError_t attn_tc_setup() {
   return cudaFuncSetAttribute(k_attn_tc_long, cudaFuncAttributeMaxDynamicSharedMemorySize, lt::SMEM_BYTES);
 }
 
-cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool3,
-                                const AttnTcArgs& a, int num_sms, cudaStream_t st) {
+cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv32,
+                                const CUtensorMap& tm_kv64, const CUtensorMap& tm_pool, const AttnTcArgs& a,
+                                int num_sms, cudaStream_t st) {
   if (a.n_units <= 0) return cudaSuccess;
   const int grid = a.n_units < num_sms ? a.n_units : num_sms;
-  k_attn_tc<<<grid, THREADS, SMEM_BYTES, st>>>(tm_q, tm_kv, tm_pool3, a);
+  k_attn_tc<<<grid, THREADS, SMEM_BYTES, st>>>(tm_q, tm_kv, tm_kv32, tm_kv64, tm_pool, a);
   return cudaGetLastError();
 }
 
-cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_pool3,
-                                     const AttnTcArgs& a, int num_sms, cudaStream_t st) {
+cudaError_t launch_attention_tc_long(const CUtensorMap& tm_q, const CUtensorMap& tm_kv, const CUtensorMap& tm_kv32,
+                                     const CUtensorMap& tm_kv64, const CUtensorMap& tm_pool, const AttnTcArgs& a,
+                                     int num_sms, cudaStream_t st) {
   if (a.n_units <= 0) return cudaSuccess;
   const int grid = a.n_units < num_sms ? a.n_units : num_sms;
-  k_attn_tc_long<<<grid, lt::THREADS, lt::SMEM_BYTES, st>>>(tm_q, tm_kv, tm_pool3, a);
+  k_attn_tc_long<<<grid, lt::THREADS, lt::SMEM_BYTES, st>>>(tm_q, tm_kv, tm_kv32, tm_kv64, tm_pool, a);
   return cudaGetLastError();
 }
 

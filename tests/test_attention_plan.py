@@ -4,11 +4,11 @@ dopr_debug_attention_plan returns the tiles dopr_score launches for one
 document's run of pairs (the prefix-plus-causal attention of Sec. 3.4).  The
 rule: tiles take consecutive packed tokens, at most rows_per_tile of them and
 at most 16 pairs; a tile's key columns are the prefix (rounded up to 64)
-followed by the run of packed tokens from the first token of the first pair it
-touches to its last token, rounded up to 16; a tensor-core tile keeps within
-256 key columns and ends only where the next token would break a limit; a
-long tile (no key limit) is made only when the first token alone needs more
-than 256 columns.  Checked on cases worked by hand, on invariants, and against an
+followed by one 16-aligned segment per pair it touches, each running from the
+pair's first token to the tile's last; a tensor-core tile keeps within 256
+key columns and ends only where the next token would break a limit; a long
+tile (no key limit) is made only when the first token alone needs more than
+256 columns.  Checked on cases worked by hand, on invariants, and against an
 independent greedy restatement on random runs.
 """
 import numpy as np
@@ -51,8 +51,8 @@ def reference_plan(m, tt, lens):
     def touched(lo, hi):  # pairs with a token in [lo, hi]
         return [p for p in range(len(lens)) if starts[p] <= hi and starts[p + 1] > lo]
 
-    def keys_of(lo, t):  # prefix, then the token run from the first touched pair's start to t
-        return c64(m) + c16(t + 1 - starts[touched(lo, t)[0]])
+    def keys_of(lo, t):
+        return c64(m) + sum(c16(min(starts[p + 1], t + 1) - starts[p]) for p in touched(lo, t))
 
     tiles, tok = [], 0
     while tok < total:
@@ -91,16 +91,14 @@ def test_full_prefix_makes_every_tile_long(lib):
     assert [(tb, n) for _, tb, n, _, _ in tiles] == [(0, 32), (32, 18)]
 
 
-def test_short_pairs_share_a_tile_as_one_token_run(lib):
-    # m = 0, 64 tokens per tile, pairs of 5 tokens: 13 pairs touch a full 64-token tile,
-    # whose own keys are the 64-token run itself
+def test_short_pairs_share_a_tile_up_to_the_key_budget(lib):
+    # m = 0, 64 tokens per tile, pairs of 5 tokens (16 columns each): 13 pairs touch a
+    # full 64-token tile, 208 key columns
     tiles = decode(dopr.attention_plan(0, 64, [5] * 20))
     kind, tb, n, keys, segs = tiles[0]
-    assert (kind, tb, n, keys) == (0, 0, 64, 64) and len(segs) == 13
+    assert (kind, tb, n, keys) == (0, 0, 64, 208) and len(segs) == 13
     assert segs[-1] == (4, 60)  # the 13th pair: 4 of its 5 tokens fall in the tile
-    # the next tile's run starts at that pair's first token, 4 tokens before the tile
-    kind, tb, n, keys, segs = tiles[1]
-    assert (tb, segs[0]) == (64, (5, -4)) and keys == c16(n + 4)
+    assert decode(dopr.attention_plan(0, 64, [5] * 20))[1][4][0] == (5, -4)
 
 
 def test_segment_limit_cuts_a_tile(lib):
@@ -121,7 +119,7 @@ def test_random_runs_match_the_restated_rule(lib, seed):
     tok = 0
     for kind, tb, n, keys, segs in got:
         assert tb == tok and 1 <= n <= tt and 1 <= len(segs) <= MAX_SEGS
-        assert keys == c64(m) + c16(n - segs[0][1])  # the run from the first pair's start
+        assert keys == c64(m) + sum(c16(v) for v, _ in segs)
         assert kind == 1 or keys <= MAX_KEYS
         if kind == 1:  # its first token alone is over budget: prefix + its pair's keys up to it
             assert c64(m) + c16(1 - segs[0][1]) > MAX_KEYS

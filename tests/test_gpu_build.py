@@ -102,10 +102,8 @@ def test_one_batch_equals_one_document_at_a_time():
         for l in range(SHAPE.n_layers):
             ka, va = a.read_layer(d, l, m)
             kb, vb = b.read_layer(d, l, m)
-            # documents that share attention tiles in one batch see other key positions in the
-            # 16-key MMA steps than alone: the stored states agree to rounding
-            np.testing.assert_allclose(ka.astype(np.float64), kb.astype(np.float64), rtol=2e-3, atol=2e-3)
-            np.testing.assert_allclose(va.astype(np.float64), vb.astype(np.float64), rtol=2e-3, atol=2e-3)
+            np.testing.assert_array_equal(ka.view(np.uint16), kb.view(np.uint16))
+            np.testing.assert_array_equal(va.view(np.uint16), vb.view(np.uint16))
 
 
 def test_build_errors_and_empty_prefix():
