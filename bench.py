@@ -544,7 +544,7 @@ def run_dopr(args, rank, world, local_rank, dist):
     g_bytes = sum(prof[f]["bytes"] for f in gemm_fams)
     achieved = g_flops / (g_ms / 1e3) / 1e12 if g_ms > 0 else None
     traffic = gemm_traffic_record()
-    roofline = {"bound": "tensor", "kernel": "k_gemm_tc (QKV/O/gate-up/down projections)",
+    roofline = {"bound": "tensor", "kernel": "k_gemm_pair (QKV/O/gate-up/down projections on CTA pairs)",
                 "achieved": achieved, "peak": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s",
                 "frac": (achieved / peaks["bf16_tflops_sustained"]) if achieved else None,
                 "peak_source": f"{peaks['source']} sustained bf16 (kernel timed inside a long step)",

@@ -263,6 +263,21 @@ def test_long_online_sequence_without_prefix():
     assert np.max(np.abs(got - ref)) <= TOL, np.max(np.abs(got - ref))
 
 
+@pytest.mark.parametrize("doc_len", [1024, 2048])
+def test_full_document_pointwise_scoring_at_the_document_budgets(doc_len):
+    # The uncompressed comparison at the paper's longest document budgets (Tab. 8: up to
+    # 2,048 tokens): [doc_len document tokens ; query ; score token] per pair with m = 0,
+    # several pairs sharing one document's text as the uncompressed run scores them.
+    rig = Rig(SMALL_G4, {0: 0}, seed=13, max_position=4096)
+    rng = np.random.default_rng(13 + doc_len)
+    doc = rng.integers(0, SMALL_G4.vocab, size=doc_len).astype(np.int32)
+    qts = [np.concatenate([doc, rng.integers(0, SMALL_G4.vocab, size=L).astype(np.int32)]) for L in (8, 37, 64)]
+    pairs = {"q_offsets": np.concatenate([[0], np.cumsum([len(t) for t in qts])]).astype(np.int32),
+             "q_tokens": np.concatenate(qts), "doc_ids": np.zeros(len(qts), np.int64)}
+    got, ref = rig.score(pairs), rig.oracle(pairs)
+    assert np.max(np.abs(got - ref)) <= TOL, np.max(np.abs(got - ref))
+
+
 def test_prefix_built_by_forward_pass_reproduces_full_forward():
     # Sec. 3.4 footnote: stored states are the per-layer K/V of forwarding the
     # prefix inputs.  Build them with the oracle, store them in bf16, and the
