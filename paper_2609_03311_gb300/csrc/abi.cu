@@ -141,6 +141,11 @@ bool kind_is_global(int32_t k) {
   return k == DOPR_W_EMBED || k == DOPR_W_FINAL_NORM || k == DOPR_W_SCORE_HEAD;
 }
 
+void free_store(Store* s) {
+  dev_free(s->pool); dev_free(s->d_slot_of); dev_free(s->d_slot_m); dev_free(s->d_slot_row); dev_free(s->d_slot_ok);
+  dev_free(s->d_range);
+}
+
 void free_workspace(Workspace& w) {
   dev_free(w.r); dev_free(w.xn); dev_free(w.qkv); dev_free(w.o); dev_free(w.act);
   dev_free(w.ss_e); dev_free(w.ss_a); dev_free(w.ss_m); dev_free(w.r_s); dev_free(w.ss_s);
@@ -150,6 +155,11 @@ void free_workspace(Workspace& w) {
   dev_free(w.items); dev_free(w.tiles); dev_free(w.err);
   host_free(w.h_tok_off); host_free(w.h_sorted_slot); host_free(w.h_err); host_free(w.h_items);
   host_free(w.h_tiles);
+  dev_free(w.sel_A); dev_free(w.sel_a_off); dev_free(w.sel_u); dev_free(w.sel_pos); dev_free(w.sel_x);
+  if (w.sel_empty) {
+    free_store(w.sel_empty);
+    delete static_cast<dopr_store*>(w.sel_empty);
+  }
   w = Workspace{};
 }
 
@@ -161,11 +171,6 @@ void free_model(Model* m) {
   free_workspace(m->ws);
   for (cudaEvent_t e : m->prof.events) cudaEventDestroy(e);
   m->prof.events.clear();
-}
-
-void free_store(Store* s) {
-  dev_free(s->pool); dev_free(s->d_slot_of); dev_free(s->d_slot_m); dev_free(s->d_slot_row); dev_free(s->d_slot_ok);
-  dev_free(s->d_range);
 }
 
 dopr_status build_weight_maps(Model* m) {
@@ -211,6 +216,20 @@ dopr_status alloc_chunk_buffers(Model* m, int cap) {
   return DOPR_OK;
 }
 
+// Grow a device buffer to at least `need` elements (at least doubling); the
+// capacity reads 0 while the buffer is not allocated, so a failed growth is
+// retried by the next call instead of leaving a stale capacity.
+template <typename T>
+dopr_status grow_dev(T** p, int64_t& cap, int64_t need) {
+  if (need <= cap) return DOPR_OK;
+  const int64_t n = std::max<int64_t>(need, 2 * cap);
+  dev_free(*p);
+  cap = 0;
+  STATUS_TRY(dev_alloc(p, (size_t)n));
+  cap = n;
+  return DOPR_OK;
+}
+
 // Grow the per-call buffers.
 dopr_status ensure_call_buffers(Model* m, int64_t n_pairs, int64_t n_tokens, int64_t n_qtokens, int64_t n_docs) {
   Workspace& w = m->ws;
@@ -218,6 +237,7 @@ dopr_status ensure_call_buffers(Model* m, int64_t n_pairs, int64_t n_tokens, int
     const int64_t cap = std::max<int64_t>(n_pairs, 2 * w.pair_cap);
     dev_free(w.q_off); dev_free(w.doc_ids); dev_free(w.scores); dev_free(w.pair_slot); dev_free(w.perm);
     dev_free(w.sorted_slot); dev_free(w.tok_off); dev_free(w.items);
+    w.pair_cap = w.item_cap = 0;  // stays 0 if the growth fails, so no later call uses a freed buffer
     STATUS_TRY(dev_alloc(&w.q_off, cap + 1));
     STATUS_TRY(dev_alloc(&w.doc_ids, cap));
     STATUS_TRY(dev_alloc(&w.scores, cap));
@@ -232,6 +252,7 @@ dopr_status ensure_call_buffers(Model* m, int64_t n_pairs, int64_t n_tokens, int
   if (n_pairs > w.h_pair_cap) {
     const int64_t cap = std::max<int64_t>(n_pairs, 2 * w.h_pair_cap);
     host_free(w.h_tok_off); host_free(w.h_sorted_slot); host_free(w.h_items);
+    w.h_pair_cap = w.h_item_cap = 0;
     STATUS_TRY(host_alloc(&w.h_tok_off, cap + 1));
     STATUS_TRY(host_alloc(&w.h_sorted_slot, cap));
     STATUS_TRY(host_alloc(&w.h_items, 2 * (cap + 1024)));
@@ -241,6 +262,7 @@ dopr_status ensure_call_buffers(Model* m, int64_t n_pairs, int64_t n_tokens, int
   if (n_tokens > w.tok_cap) {
     const int64_t cap = std::max<int64_t>(n_tokens, 2 * w.tok_cap);
     dev_free(w.tok_id); dev_free(w.tok_pos); dev_free(w.tok_pair);
+    w.tok_cap = 0;
     STATUS_TRY(dev_alloc(&w.tok_id, cap));
     STATUS_TRY(dev_alloc(&w.tok_pos, cap));
     STATUS_TRY(dev_alloc(&w.tok_pair, cap));
@@ -250,6 +272,7 @@ dopr_status ensure_call_buffers(Model* m, int64_t n_pairs, int64_t n_tokens, int
     const int64_t cap = std::max<int64_t>(n_tokens, 2 * w.tile_cap);
     dev_free(w.tiles);
     host_free(w.h_tiles);
+    w.tile_cap = 0;
     STATUS_TRY(dev_alloc(&w.tiles, cap));
     STATUS_TRY(host_alloc(&w.h_tiles, cap));
     w.tile_cap = cap;
@@ -257,11 +280,13 @@ dopr_status ensure_call_buffers(Model* m, int64_t n_pairs, int64_t n_tokens, int
   if (n_qtokens > w.qtok_cap) {
     const int64_t cap = std::max<int64_t>(n_qtokens, 2 * w.qtok_cap);
     dev_free(w.q_tok);
+    w.qtok_cap = 0;
     STATUS_TRY(dev_alloc(&w.q_tok, cap));
     w.qtok_cap = cap;
   }
   if (n_docs > w.doc_cap) {
     dev_free(w.doc_count);
+    w.doc_cap = 0;
     STATUS_TRY(dev_alloc(&w.doc_count, n_docs));
     w.doc_cap = n_docs;
   }
@@ -1329,14 +1354,12 @@ dopr_status dopr_select_prefix_inputs(dopr_model* m, int32_t n_docs, const int32
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   Workspace& w = m->ws;
   // a store of one empty document gives the attention kernels a valid pool map
-  dopr_store* empty = nullptr;
-  STATUS_TRY(dopr_store_create(&c, 0, 256, &empty));
-  // freed on return without touching this thread's error message (dopr_store_destroy clears it)
-  std::unique_ptr<dopr_store, void (*)(dopr_store*)> hold(empty, [](dopr_store* x) {
-    cudaSetDevice(x->device);
-    free_store(x);
-    delete x;
-  });
+  // (made once per model and kept, like the selection buffers below)
+  if (!w.sel_empty) {
+    dopr_store* empty = nullptr;
+    STATUS_TRY(dopr_store_create(&c, 0, 256, &empty));
+    w.sel_empty = empty;
+  }
   dopr_status rs = ensure_call_buffers(m, n_docs, T, 0, 0);
   if (rs != DOPR_OK) return rs;
   std::vector<int32_t> tok_pos(T), tok_pair(T);
@@ -1380,19 +1403,16 @@ dopr_status dopr_select_prefix_inputs(dopr_model* m, int32_t n_docs, const int32
     s0 = s1;
   }
   STATUS_TRY(ap.upload(w, plan, 0, st));
-  // selection buffers for this call
-  SelectState sel{top_k, top_p, nullptr, a_max, nullptr, nullptr, nullptr, nullptr};
-  auto cleanup = [&] {
-    dev_free(sel.A); dev_free(sel.a_off); dev_free(sel.u); dev_free(sel.positions); dev_free(sel.x);
-  };
-  if (dev_alloc(&sel.A, (size_t)a_max) != DOPR_OK || dev_alloc(&sel.a_off, (size_t)docs_max) != DOPR_OK ||
-      dev_alloc(&sel.u, (size_t)T) != DOPR_OK || dev_alloc(&sel.positions, (size_t)n_docs * top_k) != DOPR_OK ||
-      dev_alloc(&sel.x, (size_t)n_docs * top_k * H) != DOPR_OK) {
-    cleanup();
-    return fail(DOPR_ERR_OUT_OF_MEMORY, "selection buffers");
-  }
+  // selection buffers, grown on demand and kept for the next call
+  STATUS_TRY(grow_dev(&w.sel_A, w.sel_a_cap, a_max));
+  STATUS_TRY(grow_dev(&w.sel_a_off, w.sel_doc_cap, docs_max));
+  STATUS_TRY(grow_dev(&w.sel_u, w.sel_tok_cap, T));
+  STATUS_TRY(grow_dev(&w.sel_pos, w.sel_pos_cap, (int64_t)n_docs * top_k));
+  STATUS_TRY(grow_dev(&w.sel_x, w.sel_x_cap, (int64_t)n_docs * top_k * H));
+  SelectState sel{top_k, top_p, w.sel_A, a_max, w.sel_a_off, w.sel_u, w.sel_pos, w.sel_x};
   cudaError_t e = cudaMemsetAsync(w.err, 0, sizeof(int), st);
-  rs = e == cudaSuccess ? run_layers(m, empty, plan, nullptr, st, nullptr, &sel) : fail(DOPR_ERR_CUDA, "memset failed");
+  rs = e == cudaSuccess ? run_layers(m, w.sel_empty, plan, nullptr, st, nullptr, &sel)
+                         : fail(DOPR_ERR_CUDA, "memset failed");
   if (rs == DOPR_OK) {
     e = cudaMemcpyAsync(positions, sel.positions, sizeof(int32_t) * n_docs * top_k, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess)
@@ -1404,7 +1424,6 @@ dopr_status dopr_select_prefix_inputs(dopr_model* m, int32_t n_docs, const int32
   } else {
     cudaStreamSynchronize(st);
   }
-  cleanup();
   STATUS_TRY(rs);
   return map_device_error(*w.h_err);
 }

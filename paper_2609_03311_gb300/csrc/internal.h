@@ -122,6 +122,14 @@ struct Workspace {
   AttnItem* h_items = nullptr;
   AttnTile* h_tiles = nullptr;
   int64_t h_pair_cap = 0, h_item_cap = 0;
+  // key token selection (dopr_select_prefix_inputs), grown on demand and kept
+  Store* sel_empty = nullptr;  // a store of one empty document: a valid pool map for the attention kernels
+  float* sel_A = nullptr;      // per-document attention matrices of the largest chunk (sum of n^2)
+  int64_t* sel_a_off = nullptr;
+  float* sel_u = nullptr;      // salience of every token
+  int32_t* sel_pos = nullptr;  // [docs][top_k]
+  bf16* sel_x = nullptr;       // [docs][top_k][H]
+  int64_t sel_a_cap = 0, sel_doc_cap = 0, sel_tok_cap = 0, sel_pos_cap = 0, sel_x_cap = 0;
 };
 
 // Per-kernel-family launch counters and (when enabled) CUDA-event timing.

@@ -149,3 +149,25 @@ def test_select_errors():
             dopr.select_prefix_inputs(model, off, tok, K, p)
         assert ei.value.status == dopr.ERR_INVALID_ARG
     model.close()
+
+
+def test_selection_workspace_is_reused_across_calls():
+    # The n^2 attention matrices, salience, positions and states live in a
+    # workspace of the model that grows on demand and is kept.  A long call,
+    # shorter ones after it (a larger, stale workspace) and a longer one again
+    # (growth) must each return exactly what a fresh model returns.
+    shape = SHAPE_G2
+    w = synth.make_weights(shape, seed=45, norms="random")
+    cfg = dopr.make_config(shape, max_position=4096)
+    model = dopr.Model(cfg, w)
+    calls = [([300, 200, 17], 24, 4), ([5, 1], 8, 10 ** 6), ([64], 64, 2), ([900, 3, 512], 32, 1)]
+    for i, (lens, K, p) in enumerate(calls):
+        off, tok, _ = _docs(shape, lens, seed=45 + i)
+        got = dopr.select_prefix_inputs(model, off, tok, K, p)
+        fresh = dopr.Model(cfg, w)
+        want = dopr.select_prefix_inputs(fresh, off, tok, K, p)
+        fresh.close()
+        np.testing.assert_array_equal(got[0], want[0], err_msg=f"call {i}: positions")
+        assert torch.equal(got[1].view(torch.int16), want[1].view(torch.int16)), f"call {i}: states"
+        np.testing.assert_array_equal(got[2], want[2], err_msg=f"call {i}: salience")
+    model.close()
