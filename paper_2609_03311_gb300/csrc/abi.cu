@@ -483,7 +483,13 @@ struct AttnPlanner {
       tok += n;
     }
   }
-  void close_chunk(Plan& plan) const {
+  // The chunk's tiles go out most key columns first: CTAs take units round robin, so the
+  // cheapest units come last and the CTAs finish together.  A row's result does not
+  // depend on the order (each tile is computed on its own).
+  void close_chunk(Plan& plan) {
+    auto by_keys = [](const AttnTile& x, const AttnTile& y) { return x.n_keys > y.n_keys; };
+    std::stable_sort(tiles.begin() + plan.chunk_tile.back(), tiles.end(), by_keys);
+    std::stable_sort(ltiles.begin() + plan.chunk_ltile.back(), ltiles.end(), by_keys);
     plan.chunk_litem.push_back((int32_t)litems.size());
     plan.chunk_tile.push_back((int32_t)tiles.size());
     plan.chunk_ltile.push_back((int32_t)ltiles.size());
