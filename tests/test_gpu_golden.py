@@ -52,7 +52,7 @@ def _model(shape):
     return _MODELS[shape.name]
 
 
-@pytest.mark.parametrize("name", ["qwen3-8b-m64", "qwen3-8b-zipf"])
+@pytest.mark.parametrize("name", ["qwen3-8b-m64", "qwen3-8b-zipf", "qwen3-4b"])
 def test_full_size_scores_match_stored_oracle(name):
     rec = _load(name)
     wl = synth.WORKLOADS[name]
