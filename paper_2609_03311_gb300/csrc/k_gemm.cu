@@ -24,11 +24,12 @@
 //               access is a 128-byte row segment written by 8 consecutive
 //               lanes; finally tell the leader the accumulator is free, so the
 //               next tile's MMAs overlap the epilogue.
-// Tiles are visited in groups of pair-row blocks whose activation rows (up to 48 MiB:
-// 4,096 rows at K = 4,096, 2,048 at K = 12,288) stay in L2 while the weight tiles
-// stream past them.  Groups of 2,048 rows at every K streamed the weights twice as
-// often from HBM (gate/up: 3.5 GB read per 26,800-row launch instead of 1.9), and
-// under the power cap that traffic cost about 1 % of SM clock and throughput.
+// Tiles are visited in L2 groups (pair_tile_order): blocks of activation rows (up to
+// 48 MiB: 4,096 rows at K = 4,096) that stay in L2 while the weight tiles stream past
+// them, or, for the residual-epilogue launches, blocks of weight columns while the
+// activations stream.  Groups of 2,048 activation rows at every K streamed the weights
+// twice as often from HBM (gate/up: 3.5 GB read per 26,800-row launch instead of 1.9),
+// and under the power cap that traffic cost about 1 % of SM clock and throughput.
 //
 // Fused epilogues (the decoder's RMSNorms live here, not in separate kernels):
 //   RMSNorm(r) * g = rs * (r (.) g) with rs = rsqrt(mean(r^2) + eps).  The
@@ -377,12 +378,22 @@ constexpr int PAIR_STAGES = 6;
 constexpr int PAIR_B_BYTES = BM * BK * 2;       // this CTA's 128 of the tile's 256 B rows: 16 KiB
 constexpr int PAIR_STAGE_BYTES = A_BYTES + PAIR_B_BYTES;
 constexpr int PAIR_SMEM_BYTES = 1024 + PAIR_STAGES * PAIR_STAGE_BYTES + XPOSE_BYTES + BAR_BYTES;
-// Tiles go out in groups of pair-row blocks sharing their A rows in L2: as many blocks
-// as keep the group's A rows within GROUP_A_BYTES (4 to 16 blocks).
-constexpr int64_t GROUP_A_BYTES = 48ll << 20;
-__device__ __forceinline__ int pair_group_m(int K) {
-  const int64_t g = GROUP_A_BYTES / (static_cast<int64_t>(K) * 2 * 2 * BM);  // A bytes of one pair-row block
-  return g < 4 ? 4 : g > 16 ? 16 : static_cast<int>(g);
+// L2 tile groups.  A 256-row block of A and a 256-row block of B hold the same bytes
+// (256 K 2); a group holds as many blocks as fit GROUP_BYTES (row groups at most 16).
+// Row groups keep blocks of A in L2 while B streams past (once per group); column
+// groups keep blocks of B while A streams.  Measured DRAM reads per 26,800-row launch
+// (row / column groups): QKV 0.76 / 0.78 GB, O 1.31 / 1.07, gate/up 1.95 / 2.74, down
+// 3.93 / 3.12: the launches whose epilogue streams the fp32 residual (O, down) keep
+// their weight columns better, the others their activation rows.
+constexpr int64_t GROUP_BYTES = 48ll << 20;
+struct TileOrder {
+  int group;   // blocks per group
+  bool by_n;   // column groups
+};
+__device__ __forceinline__ TileOrder pair_tile_order(int n_tiles, int K, bool by_n) {
+  const int64_t g = GROUP_BYTES / (static_cast<int64_t>(K) * 2 * 2 * BM);
+  const int64_t cap = by_n ? n_tiles : 16;
+  return TileOrder{g < 1 ? 1 : g > cap ? static_cast<int>(cap) : static_cast<int>(g), by_n};
 }
 constexpr uint32_t PAIR_IDESC = umma_idesc_f16(PAIR_BM, BN);
 // TMEM columns a pair CTA allocates, and accumulators (256 columns each) it cycles through
@@ -390,14 +401,26 @@ constexpr int PAIR_ACCS = 2;
 constexpr uint32_t PAIR_TMEM_COLS = PAIR_ACCS * BN;
 static_assert(PAIR_SMEM_BYTES <= 227 * 1024, "shared memory budget");
 
-__device__ __forceinline__ void pair_tile_coords(int t, int m_tiles, int n_tiles, int group_m, int& mb, int& nb) {
-  const int group = group_m * n_tiles;
-  const int g = t / group;
-  const int first_m = g * group_m;
-  const int gm = min(group_m, m_tiles - first_m);
-  const int r = t - g * group;
-  mb = first_m + r % gm;
-  nb = r / gm;
+// Tile t of the launch: within a group the grouped operand's blocks vary fastest, so the
+// tiles of one wave share the streamed operand's blocks too.
+__device__ __forceinline__ void pair_tile_coords(int t, int m_tiles, int n_tiles, TileOrder o, int& mb, int& nb) {
+  if (o.by_n) {
+    const int group = o.group * m_tiles;
+    const int g = t / group;
+    const int first_n = g * o.group;
+    const int gn = min(o.group, n_tiles - first_n);
+    const int r = t - g * group;
+    nb = first_n + r % gn;
+    mb = r / gn;
+  } else {
+    const int group = o.group * n_tiles;
+    const int g = t / group;
+    const int first_m = g * o.group;
+    const int gm = min(o.group, m_tiles - first_m);
+    const int r = t - g * group;
+    mb = first_m + r % gm;
+    nb = r / gm;
+  }
 }
 
 template <int EPI>
@@ -423,7 +446,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   const bool leader = rank == 0;
   const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
   const int m_tiles = (p.M + PAIR_BM - 1) / PAIR_BM, n_tiles = p.N / BN, k_blocks = p.K / BK;
-  const int group_m = pair_group_m(p.K);
+  const TileOrder order = pair_tile_order(n_tiles, p.K, EPI == EPI_RESID_ADD);
   int total = m_tiles * n_tiles;
 
   if (threadIdx.x == 0) {
@@ -467,7 +490,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       bool ok = true;
       for (int t = pair; t < total && ok; t += n_pairs) {
         int mb, nb;
-        pair_tile_coords(t, m_tiles, n_tiles, group_m, mb, nb);
+        pair_tile_coords(t, m_tiles, n_tiles, order, mb, nb);
         for (int kb = 0; kb < k_blocks; ++kb) {
           if (!mbar_wait_cluster(empty_bar(stage), phase ^ 1u, p.err, p.timeout_ns)) {
             ok = false;
@@ -538,7 +561,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     int local = 0;
     for (int t = pair; t < total; t += n_pairs, ++local) {
       int mb2, nb;
-      pair_tile_coords(t, m_tiles, n_tiles, group_m, mb2, nb);
+      pair_tile_coords(t, m_tiles, n_tiles, order, mb2, nb);
       const int mb = 2 * mb2 + static_cast<int>(rank);  // this CTA's 128-row block
       const int acc = local % PAIR_ACCS;
       const uint32_t acc_phase = (local / PAIR_ACCS) & 1;
