@@ -60,7 +60,10 @@ constexpr int XPOSE_WORDS = 32 * 33;  // per epilogue warp: 32 rows x 32 words, 
 constexpr int XPOSE_BYTES = EPI_WARPS * XPOSE_WORDS * 4;
 constexpr int BAR_BYTES = 256;
 
-__device__ __forceinline__ float silu_f(float x) { return x / (1.0f + __expf(-x)); }
+// silu(x) = x / (1 + e^-x) with the fast division (within 2 ulp of fp32, far below the fp16
+// rounding of the output; tends to 0 as x -> -inf): the exact division's instruction
+// sequence made the SwiGLU epilogue outlast short main loops (K = 1,024).
+__device__ __forceinline__ float silu_f(float x) { return __fdividef(x, 1.0f + __expf(-x)); }
 
 // RMSNorm factor of a row from its partial sums of squares, added in index
 // order.  When the count allows, the partials arrive as independent 16-byte
