@@ -483,11 +483,12 @@ struct AttnPlanner {
       tok += n;
     }
   }
-  // The chunk's tiles go out most key columns first: CTAs take units round robin, so the
-  // cheapest units come last and the CTAs finish together.  A row's result does not
-  // depend on the order (each tile is computed on its own).
+  // The chunk's tiles go out most 64-key blocks first: CTAs take units round robin, so the
+  // cheapest units come last and the CTAs finish together; within a block count the
+  // tiles keep their order, so a document's tiles stay together and its prefix is read
+  // from L2.  A row's result does not depend on the order (each tile is computed on its own).
   void close_chunk(Plan& plan) {
-    auto by_keys = [](const AttnTile& x, const AttnTile& y) { return x.n_keys > y.n_keys; };
+    auto by_keys = [](const AttnTile& x, const AttnTile& y) { return (x.n_keys + 63) / 64 > (y.n_keys + 63) / 64; };
     std::stable_sort(tiles.begin() + plan.chunk_tile.back(), tiles.end(), by_keys);
     std::stable_sort(ltiles.begin() + plan.chunk_ltile.back(), ltiles.end(), by_keys);
     plan.chunk_litem.push_back((int32_t)litems.size());
